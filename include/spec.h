@@ -1,0 +1,230 @@
+/*
+ * spec.h -- C ABI of the GB300 batched speculative-verification library
+ * (libspec.so, built for sm_103a).
+ *
+ * One decoding round of the method of arxiv 2607.25852 ("AngelSpec"):
+ *   spec_allocate  D-cut batch-level verification-depth allocation and dense
+ *                  packing (Section 4.2: Eqs. dcut-score, dcut-expected-advance,
+ *                  dcut-budget, dcut-batch-utility, dcut-select; "Packing and
+ *                  correctness").
+ *   spec_verify    target verification of the packed drafts by rejection
+ *                  sampling (Section 1; Eq. mtp-acceptance-tv in Section 2;
+ *                  the deterministic-draft, target-only protocol of Section
+ *                  4.2), with temperature 0 as the longest argmax prefix.
+ *   spec_commit    packing of the committed tokens and of the target hidden
+ *                  rows that condition the drafter's next round (Sections 1,
+ *                  3.1 and 6).
+ *
+ * Conventions shared by every entry point
+ *   - Pointers marked "device" are CUDA device (or managed) memory of the
+ *     current device; "host" pointers are ordinary host memory read during
+ *     the call.  The caller owns every buffer.  The library never allocates
+ *     device memory, never synchronises the stream and never reads device
+ *     memory on the host, so every call is stream-ordered on `stream`.
+ *   - Argument errors that the host can see return a spec_err code
+ *     synchronously and launch nothing.  Data errors found on the device
+ *     (bad token ids, NaN logits, confidences outside [0,1], inconsistent
+ *     offsets) are reported through `status`, a device int32 that the caller
+ *     zero-fills beforehand: the first error code wins (atomic
+ *     compare-and-swap), the kernels still run to completion, and the
+ *     affected request's outputs are set to defined values (accepted length
+ *     0, tokens -1).  No kernel traps or asserts.
+ *   - A device-side wait never spins without a bound.
+ *   - Element types: SPEC_BF16 (IEEE binary32 truncated to its upper 16 bits)
+ *     or SPEC_F32.
+ *
+ * Random numbers (a reading: the paper does not fix a generator).  Every
+ * uniform is drawn from Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11)
+ * with key = (lo32(seed_i), hi32(seed_i)) and counter =
+ *   (lo32(position), lo32(request_id_i), hi32(request_id_i), purpose<<28 | sub)
+ *   SPEC_PURPOSE_ACCEPT: sub = 0; u = (word0 >> 8) * 2^-24 in [0, 1)
+ *   SPEC_PURPOSE_SAMPLE: sub = v >> 2; E_v = -ln(((word[v & 3] >> 8) + 1) * 2^-24)
+ * so a round replays bit for bit from (seed, request id, position).
+ */
+#ifndef SPEC_H_
+#define SPEC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SPEC_ABI_VERSION 1
+
+typedef enum {
+  SPEC_OK = 0,
+  SPEC_ERR_INVALID_ARG = 1, /* host-visible argument error; nothing launched */
+  SPEC_ERR_WORKSPACE = 2,   /* workspace missing, too small or misaligned */
+  SPEC_ERR_CUDA = 3,        /* a CUDA runtime call failed (e.g. launch) */
+  SPEC_ERR_BAD_INPUT = 4,   /* device-detected data error (via *status) */
+  SPEC_ERR_TIMEOUT = 5      /* a bounded device wait gave up (via *status) */
+} spec_err;
+
+typedef enum { SPEC_BF16 = 0, SPEC_F32 = 1 } spec_dtype;
+
+#define SPEC_PURPOSE_ACCEPT 1u
+#define SPEC_PURPOSE_SAMPLE 2u
+
+/* Limits checked on the host (SPEC_ERR_INVALID_ARG beyond them). */
+#define SPEC_MAX_VOCAB (1 << 30)       /* V < 2^30 keeps v >> 2 within 28 bits */
+#define SPEC_MAX_DRAFTS 255            /* K */
+#define SPEC_MAX_ALLOC_POSITIONS 8192  /* B(K+1) for spec_allocate */
+#define SPEC_MAX_CANDIDATES 64         /* M for spec_allocate */
+
+/* Human-readable name of a spec_err code (static string). */
+const char* spec_error_string(int code);
+
+/* SPEC_ABI_VERSION of the loaded library. */
+int spec_version(void);
+
+/* ------------------------------------------------------------------------
+ * spec_budget_from_ratios -- Eq. (dcut-budget), Section 4.2:
+ *   T_m = max(B, ceil(num[m] / den[m] * B * (K + 1)))
+ * in exact integer arithmetic, for M ratios (the paper's set is
+ * {1/4, 1/2, 3/4, 1}).  Host only.
+ *   num, den     host int32 [M]; 0 <= num[m] <= den[m], den[m] > 0.
+ *   cand_T_out   host int32 [M].
+ * Returns SPEC_OK or SPEC_ERR_INVALID_ARG.
+ * ---------------------------------------------------------------------- */
+int spec_budget_from_ratios(int B, int K, const int32_t* num, const int32_t* den,
+                            int M, int32_t* cand_T_out);
+
+/* ------------------------------------------------------------------------
+ * spec_allocate -- D-cut allocation and packing (Section 4.2).
+ *   1. s_{i,0} = 1, s_{i,k} = s_{i,k-1} * c_{i,k} as fp32 products taken in
+ *      order k = 1..K (Eq. dcut-score).
+ *   2. All B(K+1) positions are ranked by s descending, ties toward the
+ *      shallower k (the paper's rule), then toward the lower request index.
+ *   3. For each candidate budget T_m, the top-T_m positions give keep depths
+ *      n_i(T_m) (a contiguous prefix per request) and the utility
+ *      U_m = sum_i sum_{k<=n_i} s_{i,k} (Eqs. dcut-expected-advance,
+ *      dcut-batch-utility), evaluated exactly as the integer sum of
+ *      floor(s * 2^40) and reported as that sum * 2^-40.
+ *   4. The chosen budget is the first maximiser of U_m / cost_m (Eq.
+ *      dcut-select, fp64 division).
+ *   5. Packing: row_offsets = exclusive scan of (n_i + 1); packed row
+ *      row_offsets[i] + j carries token last_tokens[i] (j = 0) or
+ *      draft_tokens[i][j-1] (j >= 1) at position pos_base[i] + j.
+ * Arguments
+ *   conf            device fp32 [B, K], row-major: c_{i,k} at [i][k-1].
+ *   cand_T          host int32 [M], each in [B, B(K+1)].
+ *   cand_cost       host fp64 [M], each finite and > 0 (the profiled
+ *                   step latency C(B, rho) of the candidate).
+ *   last_tokens     device int32 [B]; draft_tokens device int32 [B, K];
+ *   pos_base        device int64 [B] (position of row 0 of each request).
+ *   depth_out       device int32 [B]; row_offsets_out device int32 [B+1];
+ *   packed_tokens_out device int32 [B(K+1)], packed_pos_out device int64
+ *                   [B(K+1)]: rows past the chosen budget are set to -1.
+ *   chosen_T_out    device int32 [1]; utility_out device fp64 [M] or NULL.
+ *   status          device int32 [1] (see conventions).
+ *   ws, ws_bytes    unused (spec_allocate_workspace returns 0); may be NULL.
+ * Limits: 1 <= B, 0 <= K <= SPEC_MAX_DRAFTS, B(K+1) <= SPEC_MAX_ALLOC_POSITIONS,
+ * 1 <= M <= SPEC_MAX_CANDIDATES.  A confidence that is NaN or outside [0, 1]
+ * counts as 0 and sets SPEC_ERR_BAD_INPUT.
+ * ---------------------------------------------------------------------- */
+size_t spec_allocate_workspace(int B, int K, int M);
+int spec_allocate(const float* conf, int B, int K, const int32_t* cand_T,
+                  const double* cand_cost, int M, const int32_t* last_tokens,
+                  const int32_t* draft_tokens, const int64_t* pos_base,
+                  int32_t* depth_out, int32_t* row_offsets_out,
+                  int32_t* packed_tokens_out, int64_t* packed_pos_out,
+                  int32_t* chosen_T_out, double* utility_out, int32_t* status,
+                  void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * spec_verify -- batched verification (Section 1: rejection sampling with
+ * the target unchanged; Eq. mtp-acceptance-tv; Section 4.2: deterministic-
+ * draft, target-only protocol when q is NULL).
+ * For request i with n = n_i kept drafts z_1..z_n and logits rows
+ * l_0..l_n (row j verifies draft z_{j+1}; row n is the bonus row):
+ *   t == 0: g_j = argmax_v l_j[v] (lowest v on ties);
+ *           a = longest prefix with z_{j+1} == g_j; y = g_a.
+ *   t  > 0: p_j = softmax(l_j / t); for j = 0..n-1 accept z_{j+1} iff
+ *           u_j < min(1, p_j(z_{j+1}) / q_j(z_{j+1}))   (q_j(z) = 0 gives 1
+ *           if p_j(z) > 0); at the first rejection a = j and y is drawn from
+ *           max(0, p_a - q_a) (from p_a if that is identically zero); if all
+ *           n are accepted, a = n and y is drawn from p_n.  The draw is the
+ *           exponential race y = argmin_{w_v > 0} E_v / w_v (lowest v on
+ *           ties), an exact sampler of w / sum(w) that does not depend on
+ *           summation order.
+ *   out_tokens[i] = z_1..z_a, y, then -1 up to K+1 entries.
+ * Arguments
+ *   logits          device [R, V] of logits_dtype, rows of request i at
+ *                   row_offsets[i] .. row_offsets[i] + n_i.
+ *   row_offsets     device int32 [B+1] (from spec_allocate) or NULL, meaning
+ *                   row_offsets[i] = i(K+1) and R = B(K+1).
+ *   depth           device int32 [B] (n_i in [0, K]) or NULL meaning n_i = K.
+ *                   If row_offsets is given, row_offsets[i+1] - row_offsets[i]
+ *                   must equal n_i + 1 (else SPEC_ERR_BAD_INPUT for i).
+ *   draft_tokens    device int32 [B, K] (z_{j+1} at [i][j]); may be NULL if K=0.
+ *   q               device [B, K, V] of q_dtype (row j of request i is the
+ *                   drafter's distribution of z_{j+1}, used as stored), or
+ *                   NULL: one-hot at the draft token.  Ignored when t == 0.
+ *   temperature     t >= 0 and finite.
+ *   seeds, request_ids  device uint64 [B]; pos_base device int64 [B]
+ *                   (position of row 0; pos_base + n_i < 2^32).
+ *   accepted_len_out device int32 [B]; out_tokens device int32 [B, K+1].
+ *   p_draft_out     device fp32 [B, K] or NULL: p_j(z_{j+1}) for j < n_i
+ *                   (at t == 0: 1 if z_{j+1} == g_j else 0); other entries 0.
+ *   row_stats_out   device fp32 [B(K+1), 2] or NULL: per packed row,
+ *                   (max_v l/t, ln sum_v exp(l/t - max)); (max_v l, 0) at t == 0.
+ *   status          device int32 [1].
+ *   ws, ws_bytes    device workspace of at least spec_verify_workspace(B, K, V)
+ *                   bytes, 256-byte aligned, zero-filled once before its first
+ *                   use; the library leaves it zeroed again after each call.
+ *                   Calls that may overlap on the device need separate
+ *                   workspaces.
+ * Limits: 1 <= B, 0 <= K <= SPEC_MAX_DRAFTS, 1 <= V < SPEC_MAX_VOCAB,
+ * logits rows and q rows addressed with 64-bit offsets.
+ * ---------------------------------------------------------------------- */
+size_t spec_verify_workspace(int B, int K, int V);
+int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets,
+                const int32_t* depth, const int32_t* draft_tokens, const void* q,
+                int q_dtype, int B, int K, int V, float temperature,
+                const uint64_t* seeds, const uint64_t* request_ids,
+                const int64_t* pos_base, int32_t* accepted_len_out,
+                int32_t* out_tokens, float* p_draft_out, float* row_stats_out,
+                int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * spec_commit -- pack the committed round for the drafter's next step
+ * (Section 1: the verified prefix plus one target token is committed;
+ * Sections 3.1 and 6: the drafter conditions on target hidden states).
+ *   commit_offsets[i] = sum_{i' < i} (a_{i'} + 1), commit_offsets[B] = total.
+ *   packed_tokens_out[commit_offsets[i] + j] = out_tokens[i][j], j = 0..a_i.
+ *   hidden_out[commit_offsets[i] + j] = hidden[row_offsets[i] + j], j = 0..a_i
+ *   (the target states of the context positions that are now committed).
+ * Arguments
+ *   accepted_len, out_tokens  device int32 [B], [B, K+1] (from spec_verify).
+ *   row_offsets     device int32 [B+1] or NULL (= i(K+1)).
+ *   hidden          device [R, H] of hidden_dtype, or NULL (tokens only).
+ *   packed_tokens_out device int32 [B(K+1)] (entries past the total are
+ *                   not written); commit_offsets_out device int32 [B+1];
+ *   hidden_out      device [B(K+1), H] (worst case) or NULL.
+ *   status          device int32 [1]; an accepted length outside [0, K] sets
+ *                   SPEC_ERR_BAD_INPUT and is treated as 0.
+ * ---------------------------------------------------------------------- */
+int spec_commit(const int32_t* accepted_len, const int32_t* out_tokens,
+                const int32_t* row_offsets, const void* hidden, int hidden_dtype,
+                int B, int K, int H, int32_t* packed_tokens_out,
+                int32_t* commit_offsets_out, void* hidden_out, int32_t* status,
+                cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * spec_profile_stream_pass -- measurement aid.  The next spec_verify call
+ * records `before` immediately before and `after` immediately after its
+ * vocabulary-streaming kernel, on its stream, then forgets both.  Arguments
+ * are cudaEvent_t handles created by the caller (NULL, NULL cancels).
+ * Not thread-safe: meant for a single benchmarking thread.
+ * ---------------------------------------------------------------------- */
+int spec_profile_stream_pass(cudaEvent_t before, cudaEvent_t after);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPEC_H_ */

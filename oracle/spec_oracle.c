@@ -278,6 +278,8 @@ int oracle_verify_request(const void* logits, int logits_dtype,
     if (row_logS_out) row_logS_out[j] = log(S[j]);
   }
 
+  /* Acceptance test of every kept draft; the chain stops at the first
+   * rejection (later drafts are reported but do not matter). */
   int a = n;
   int rejected = 0;
   for (int j = 0; j < n; ++j) {
@@ -297,10 +299,9 @@ int oracle_verify_request(const void* logits, int logits_dtype,
     if (p_draft_out) p_draft_out[j] = pz;
     if (u_out) u_out[j] = u;
     if (r_out) r_out[j] = r;
-    if (!(u < r)) {
+    if (!rejected && !(u < r)) {
       a = j;
       rejected = 1;
-      break;
     }
   }
 

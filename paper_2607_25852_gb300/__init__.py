@@ -1,0 +1,159 @@
+"""GB300 (sm_103a) batched speculative verification: Python binding of libspec.
+
+The functions below carry the names of the C ABI in ``include/spec.h`` and do
+argument marshalling only (torch tensors -> device pointers, the current torch
+stream -> cudaStream_t, error codes -> exceptions).  Every step of the path runs
+in the CUDA kernels of ``libspec.so``; there is no CPU fallback.
+
+Round of arxiv 2607.25852 (AngelSpec): ``spec_allocate`` (D-cut, Section 4.2)
+-> target forward over the packed rows (caller) -> ``spec_verify`` (rejection
+sampling, Section 1) -> ``spec_commit`` (packing for the next drafting step).
+"""
+import ctypes
+
+import torch
+
+from . import _native
+
+BF16 = 0
+F32 = 1
+
+OK = 0
+ERR_INVALID_ARG = 1
+ERR_WORKSPACE = 2
+ERR_CUDA = 3
+ERR_BAD_INPUT = 4
+ERR_TIMEOUT = 5
+
+MAX_DRAFTS = 255
+MAX_ALLOC_POSITIONS = 8192
+MAX_CANDIDATES = 64
+
+__all__ = [
+    "SpecError", "spec_version", "spec_error_string", "spec_budget_from_ratios",
+    "spec_allocate_workspace", "spec_allocate", "spec_verify_workspace", "spec_verify",
+    "spec_commit", "spec_profile_stream_pass", "verify_workspace", "library",
+]
+
+
+class SpecError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {spec_error_string(code)} (code {code})")
+
+
+def library():
+    """The loaded ctypes handle of libspec.so."""
+    return _native.load()
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch.Tensor or None")
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to libspec must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype(t):
+    if t is None:
+        return BF16
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError(f"unsupported element type {t.dtype} (bf16 or fp32)")
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(code, where):
+    if code != OK:
+        raise SpecError(code, where)
+
+
+def spec_version() -> int:
+    return library().spec_version()
+
+
+def spec_error_string(code: int) -> str:
+    return library().spec_error_string(code).decode()
+
+
+def spec_budget_from_ratios(B: int, K: int, num, den):
+    """Eq. (dcut-budget) for ratios num/den; host integers in, list out."""
+    M = len(num)
+    n = (ctypes.c_int32 * M)(*num)
+    d = (ctypes.c_int32 * M)(*den)
+    out = (ctypes.c_int32 * M)()
+    _check(library().spec_budget_from_ratios(B, K, n, d, M, out), "spec_budget_from_ratios")
+    return list(out)
+
+
+def spec_allocate_workspace(B: int, K: int, M: int) -> int:
+    return library().spec_allocate_workspace(B, K, M)
+
+
+def spec_allocate(conf, cand_T, cand_cost, last_tokens, draft_tokens, pos_base, depth_out,
+                  row_offsets_out, packed_tokens_out, packed_pos_out, chosen_T_out,
+                  utility_out=None, status=None, ws=None, stream=None):
+    """conf [B, K] fp32 device; cand_T / cand_cost host sequences; see spec.h."""
+    B, K = conf.shape
+    M = len(cand_T)
+    T = (ctypes.c_int32 * M)(*[int(x) for x in cand_T])
+    C = (ctypes.c_double * M)(*[float(x) for x in cand_cost])
+    code = library().spec_allocate(
+        _ptr(conf), B, K, T, C, M, _ptr(last_tokens), _ptr(draft_tokens), _ptr(pos_base),
+        _ptr(depth_out), _ptr(row_offsets_out), _ptr(packed_tokens_out), _ptr(packed_pos_out),
+        _ptr(chosen_T_out), _ptr(utility_out), _ptr(status), _ptr(ws),
+        0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+    _check(code, "spec_allocate")
+
+
+def spec_verify_workspace(B: int, K: int, V: int) -> int:
+    return library().spec_verify_workspace(B, K, V)
+
+
+def verify_workspace(B: int, K: int, V: int, device="cuda"):
+    """A zero-filled workspace tensor of the size spec_verify needs."""
+    n = spec_verify_workspace(B, K, V)
+    if n == 0:
+        raise SpecError(ERR_INVALID_ARG, "spec_verify_workspace")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def spec_verify(logits, draft_tokens, q, B, K, V, temperature, seeds, request_ids, pos_base,
+                accepted_len_out, out_tokens, ws, row_offsets=None, depth=None, p_draft_out=None,
+                row_stats_out=None, status=None, stream=None):
+    """logits [R, V] bf16/fp32, q [B, K, V] or None; seeds/request_ids int64 (uint64 bits)."""
+    code = library().spec_verify(
+        _ptr(logits), _dtype(logits), _ptr(row_offsets), _ptr(depth), _ptr(draft_tokens),
+        _ptr(q), _dtype(q), B, K, V, float(temperature), _ptr(seeds), _ptr(request_ids),
+        _ptr(pos_base), _ptr(accepted_len_out), _ptr(out_tokens), _ptr(p_draft_out),
+        _ptr(row_stats_out), _ptr(status), _ptr(ws), ws.numel() * ws.element_size(),
+        _stream(stream))
+    _check(code, "spec_verify")
+
+
+def spec_commit(accepted_len, out_tokens, hidden, B, K, packed_tokens_out, commit_offsets_out,
+                hidden_out=None, row_offsets=None, status=None, stream=None):
+    """hidden [R, H] bf16/fp32 or None; see spec.h."""
+    H = 0 if hidden is None else hidden.shape[-1]
+    code = library().spec_commit(
+        _ptr(accepted_len), _ptr(out_tokens), _ptr(row_offsets), _ptr(hidden), _dtype(hidden),
+        B, K, H, _ptr(packed_tokens_out), _ptr(commit_offsets_out), _ptr(hidden_out),
+        _ptr(status), _stream(stream))
+    _check(code, "spec_commit")
+
+
+def spec_profile_stream_pass(before=None, after=None):
+    """Record torch.cuda.Event `before`/`after` around the next verify's streaming kernel."""
+    b = None if before is None else ctypes.c_void_p(before.cuda_event)
+    a = None if after is None else ctypes.c_void_p(after.cuda_event)
+    _check(library().spec_profile_stream_pass(b, a), "spec_profile_stream_pass")

@@ -1,0 +1,106 @@
+"""Helpers for the GPU-vs-oracle parity tests.
+
+The CUDA path is called through the C ABI (paper_2607_25852_gb300 binding);
+the oracle runs on the CPU over the very same input bytes.  Comparison rules:
+
+  * accepted lengths, committed tokens, depths, packed maps, gathered rows:
+    bit-exact;
+  * p_j(z_{j+1}) and the row statistics: relative 1e-5 (ln S: absolute 1e-5);
+  * an acceptance decision may differ only where |u - min(1, p/q)| < 1e-6
+    (the oracle's u and r); a sampled token may differ only where the oracle's
+    two best race keys are within a relative 1e-5 of each other and the GPU
+    picked the runner-up.  Each such case is counted; the rest of that request
+    is not compared bit-exactly.
+"""
+import numpy as np
+import torch
+
+import oracle
+
+P_RTOL = 1e-5
+ACCEPT_TIE = 1e-6
+RACE_TIE = 1e-5
+
+
+def bits(t):
+    t = t.detach().cpu().contiguous()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).numpy().view(np.uint16)
+    return t.numpy()
+
+
+def u64(t):
+    return t.detach().cpu().numpy().view(np.uint64)
+
+
+def run_verify(logits, drafts, q, B, K, V, t, seeds, request_ids, pos_base, row_offsets=None,
+               depth=None, ws=None, device="cuda"):
+    import paper_2607_25852_gb300 as spec
+    dev = torch.device(device)
+    d = lambda x: None if x is None else x.to(dev).contiguous()
+    ws = spec.verify_workspace(B, K, V, dev) if ws is None else ws
+    acc = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    tok = torch.full((B, K + 1), -7, dtype=torch.int32, device=dev)
+    pdr = torch.full((B, max(K, 1)), -7.0, dtype=torch.float32, device=dev)
+    rst = torch.zeros((B * (K + 1), 2), dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    spec.spec_verify(d(logits), d(drafts), d(q), B, K, V, t, d(seeds), d(request_ids), d(pos_base),
+                     acc, tok, ws, row_offsets=d(row_offsets), depth=d(depth),
+                     p_draft_out=pdr if K > 0 else None, row_stats_out=rst, status=status)
+    torch.cuda.synchronize()
+    return dict(accepted=acc.cpu().numpy(), tokens=tok.cpu().numpy(), p_draft=pdr.cpu().numpy()[:, :K],
+                row_stats=rst.cpu().numpy(), status=int(status.item()), ws=ws)
+
+
+def run_oracle(logits, drafts, q, t, seeds, request_ids, pos_base, row_offsets=None, depth=None):
+    return oracle.verify_batch(bits(logits), drafts.cpu().numpy(), None if q is None else bits(q), t,
+                               u64(seeds), u64(request_ids), pos_base.cpu().numpy(),
+                               None if row_offsets is None else row_offsets.cpu().numpy(),
+                               None if depth is None else depth.cpu().numpy())
+
+
+def compare(gpu, ref, K, t, depth=None, row_offsets=None, check_stats=True):
+    """Assert parity; returns (n_accept_ties, n_race_ties, n_positions)."""
+    B = len(ref["accepted"])
+    n_acc_ties = n_race_ties = 0
+    positions = 0
+    for i in range(B):
+        n = K if depth is None else int(depth[i])
+        positions += n + 1
+        ga, ra = int(gpu["accepted"][i]), int(ref["accepted"][i])
+        gt, rt = gpu["tokens"][i], ref["tokens"][i]
+        if ref["status"][i] != 0:
+            assert ga == 0 and (gt == -1).all(), f"request {i}: bad input not flagged"
+            continue
+        if ga != ra:
+            j = min(ga, ra)
+            assert t > 0 and j < n, f"request {i}: accepted {ga} vs oracle {ra}"
+            gap = abs(ref["u"][i, j] - ref["r"][i, j])
+            assert gap < ACCEPT_TIE, f"request {i}: decision at {j} differs, |u-r|={gap:.3g}"
+            assert gt[:j].tolist() == rt[:j].tolist()
+            n_acc_ties += 1
+            continue
+        assert gt[:ra].tolist() == rt[:ra].tolist(), f"request {i}: accepted drafts differ"
+        assert (gt[ra + 1:] == -1).all(), f"request {i}: padding"
+        if gt[ra] != rt[ra]:
+            best, bi, second, si = ref["race"][i]
+            rel = (second - best) / best if best > 0 else np.inf
+            assert t > 0 and int(si) == gt[ra] and rel < RACE_TIE, (
+                f"request {i}: token {gt[ra]} vs oracle {rt[ra]} (race gap {rel:.3g})")
+            n_race_ties += 1
+        if t > 0 and n > 0:
+            np.testing.assert_allclose(gpu["p_draft"][i, :n], ref["p_draft"][i, :n], rtol=P_RTOL,
+                                       atol=1e-30, err_msg=f"request {i}: p_draft")
+    if check_stats:
+        rows = []
+        for i in range(B):
+            if ref["status"][i] != 0:
+                continue
+            n = K if depth is None else int(depth[i])
+            row0 = i * (K + 1) if row_offsets is None else int(row_offsets[i])
+            rows.extend(range(row0, row0 + n + 1))
+        rows = np.asarray(rows, np.int64)
+        np.testing.assert_allclose(gpu["row_stats"][rows, 0], ref["row_m"][rows], rtol=P_RTOL, atol=0)
+        np.testing.assert_allclose(gpu["row_stats"][rows, 1], ref["row_logS"][rows], rtol=0, atol=P_RTOL)
+    assert n_acc_ties + n_race_ties <= max(1, 1e-4 * positions), (n_acc_ties, n_race_ties, positions)
+    return n_acc_ties, n_race_ties, positions

@@ -1,0 +1,97 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and
+loads, exports every function include/spec.h declares, and rejects bad
+arguments synchronously (before any CUDA call)."""
+import ctypes
+import os
+import re
+from fractions import Fraction
+from math import ceil
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "spec.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_25852_gb300 import build
+    build.build()
+    from paper_2607_25852_gb300 import _native
+    return _native.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(spec_[a-z_]+)\s*\(", text, re.M)
+    return sorted(set(names))
+
+
+def test_every_declared_function_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 9, names
+    from paper_2607_25852_gb300 import _native
+    assert sorted(_native.SIGNATURES) == names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_error_strings(lib):
+    import paper_2607_25852_gb300 as spec
+    assert spec.spec_version() == 1
+    assert "bad input" in spec.spec_error_string(spec.ERR_BAD_INPUT)
+    assert spec.spec_error_string(99) == "unknown error code"
+
+
+def test_budget_from_ratios_is_exact(lib):
+    import paper_2607_25852_gb300 as spec
+    for B, K in [(1, 0), (3, 0), (4, 8), (5, 8), (64, 16), (7, 255)]:
+        num, den = [1, 1, 3, 1, 0, 2, 5], [4, 2, 4, 1, 3, 3, 7]
+        got = spec.spec_budget_from_ratios(B, K, num, den)
+        want = [max(B, ceil(Fraction(n, d) * B * (K + 1))) for n, d in zip(num, den)]
+        assert got == want
+    for bad in ([1], [0]), ([2], [1]), ([-1], [2]):
+        with pytest.raises(spec.SpecError):
+            spec.spec_budget_from_ratios(4, 3, *bad)
+
+
+def test_workspace_sizes(lib):
+    import paper_2607_25852_gb300 as spec
+    assert spec.spec_verify_workspace(0, 4, 100) == 0
+    assert spec.spec_verify_workspace(4, 256, 100) == 0
+    assert spec.spec_verify_workspace(4, 4, 1 << 30) == 0
+    n = spec.spec_verify_workspace(64, 16, 201088)
+    assert n > 0 and n % 256 == 0 and n < (1 << 20)
+    assert spec.spec_allocate_workspace(64, 16, 4) == 0
+
+
+def test_argument_errors_return_before_any_launch(lib):
+    dummy = ctypes.c_void_p(16)          # never dereferenced: every call below fails its checks
+    ws = ctypes.c_void_p(256)
+    stream = ctypes.c_void_p(0)
+    v = lambda B, K, V, t, ws_bytes=1 << 20, dt=0: lib.spec_verify(
+        dummy, dt, None, None, dummy, None, 0, B, K, V, t, dummy, dummy, dummy, dummy, dummy,
+        None, None, None, ws, ws_bytes, stream)
+    assert v(0, 4, 100, 1.0) == 1
+    assert v(4, 4, 0, 1.0) == 1
+    assert v(4, 256, 100, 1.0) == 1
+    assert v(4, 4, 100, -1.0) == 1
+    assert v(4, 4, 100, float("nan")) == 1
+    assert v(4, 4, 100, float("inf")) == 1
+    assert v(4, 4, 100, 1.0, dt=7) == 1
+    assert v(4, 4, 100, 1.0, ws_bytes=8) == 2
+    assert lib.spec_verify(dummy, 0, None, None, dummy, None, 0, 4, 4, 100, 1.0, dummy, dummy, dummy,
+                           dummy, dummy, None, None, None, ctypes.c_void_p(264), 1 << 20, stream) == 2
+    a = lambda T, C, B=2, K=2: lib.spec_allocate(
+        dummy, B, K, (ctypes.c_int32 * 1)(T), (ctypes.c_double * 1)(C), 1, dummy, dummy, dummy,
+        dummy, dummy, dummy, dummy, dummy, None, None, None, 0, stream)
+    assert a(1, 1.0) == 1 and a(7, 1.0) == 1 and a(4, 0.0) == 1 and a(4, float("nan")) == 1
+    assert a(8193, 1.0, B=8193, K=0) == 1
+    c = lambda B, K, hidden, hout, H=8, dt=0: lib.spec_commit(
+        dummy, dummy, None, hidden, dt, B, K, H, dummy, dummy, hout, None, stream)
+    assert c(0, 2, None, None) == 1
+    assert c(2, 2, dummy, None) == 1
+    assert c(2, 2, dummy, dummy, H=0) == 1
+    assert c(2, 2, dummy, dummy, dt=3) == 1
+    assert lib.spec_profile_stream_pass(dummy, None) == 1
