@@ -1,0 +1,481 @@
+"""Benchmark of the batched speculative-verification hot path on GB300.
+
+One step = one round of the method over one batch of the stress workload
+(B=64 requests, K=16 drafts, V=201088 bf16 logits, bf16 q, temperature 1,
+hidden rows H=7168 bf16):
+
+    spec_allocate  D-cut over the paper's ratios {1/4, 1/2, 3/4, 1} with a flat
+                   cost table (light load: the full block wins, T* = B(K+1))
+    spec_verify    rejection-sampling verification of all 1088 rows
+    spec_commit    packing of the committed tokens and hidden rows
+
+value = verified positions per second (rows verified / step time), inputs
+resident in HBM.  The logits alone (437.6 MB) exceed L2 (126 MB), so no L2
+flush is needed between steps.  The JSON line also carries the roofline of the
+vocabulary-streaming kernel, clocks sampled during the timed region, an
+end-to-end number through the same public API with host (pinned) buffers, and
+the CPU oracle timed on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Under torchrun (N > 1) each rank runs its own batch (weak scaling, no
+collective on the data path); timing is the max over ranks.
+"""
+import argparse
+import concurrent.futures as cf
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified positions/s"
+UNIT = "positions/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="stress")
+    ap.add_argument("--V", type=int, default=None)
+    ap.add_argument("--B", type=int, default=None)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (rank layout only; no collective touches the data path)
+# ---------------------------------------------------------------------------
+def dist_info():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def dist_init(world, backend):
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    dist.init_process_group(backend=backend)
+    return dist
+
+
+def max_over_ranks(dist, value, device):
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu_index = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu_index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# the workload
+# ---------------------------------------------------------------------------
+def make_inputs(args, rank, device):
+    import torch
+    import workloads
+    wl = workloads.make(args.workload, device=device, seed=1234 + rank, V=args.V, B=args.B)
+    B, K = wl.B, wl.K
+    # Confidences for the allocator: the code/chat mix of the alloc workload.
+    rng = np.random.default_rng(4321 + rank)
+    half = B // 2
+    conf = np.concatenate([rng.beta(2.0, 2.0, (half, K)), rng.beta(8.0, 1.0, (B - half, K))])
+    wl.conf = torch.as_tensor(conf.astype(np.float32), device=device)
+    return wl
+
+
+class Step:
+    """Buffers and one call sequence allocate -> verify -> commit."""
+
+    def __init__(self, wl, device):
+        import torch
+        import paper_2607_25852_gb300 as spec
+        self.spec = spec
+        self.wl = wl
+        B, K, V = wl.B, wl.K, wl.V
+        self.ratios = spec.spec_budget_from_ratios(B, K, [1, 1, 3, 1], [4, 2, 4, 1])
+        self.costs = [1.0, 1.0, 1.0, 1.0]
+        i32, i64 = torch.int32, torch.int64
+        z = lambda *s, dt=i32: torch.zeros(s, dtype=dt, device=device)
+        self.depth, self.row_off = z(B), z(B + 1)
+        self.ptok, self.ppos = z(B * (K + 1)), z(B * (K + 1), dt=i64)
+        self.chosen = z(1)
+        self.util = z(len(self.ratios), dt=torch.float64)
+        self.acc, self.tok = z(B), z(B, K + 1)
+        self.ctok, self.coff = z(B * (K + 1)), z(B + 1)
+        self.hout = None if wl.hidden is None else torch.empty_like(wl.hidden)
+        self.status = z(1)
+        self.ws = spec.verify_workspace(B, K, V, device)
+
+    def run(self, inputs=None):
+        wl = self.wl
+        x = inputs or dict(conf=wl.conf, logits=wl.logits, drafts=wl.drafts, q=wl.q, seeds=wl.seeds,
+                           request_ids=wl.request_ids, pos_base=wl.pos_base,
+                           last_tokens=wl.last_tokens, hidden=wl.hidden)
+        s = self.spec
+        s.spec_allocate(x["conf"], self.ratios, self.costs, x["last_tokens"], x["drafts"],
+                        x["pos_base"], self.depth, self.row_off, self.ptok, self.ppos, self.chosen,
+                        self.util, self.status)
+        s.spec_verify(x["logits"], x["drafts"], x["q"], wl.B, wl.K, wl.V, wl.temperature,
+                      x["seeds"], x["request_ids"], x["pos_base"], self.acc, self.tok, self.ws,
+                      row_offsets=self.row_off, depth=self.depth, status=self.status)
+        s.spec_commit(self.acc, self.tok, x.get("hidden"), wl.B, wl.K, self.ctok, self.coff, self.hout,
+                      row_offsets=self.row_off, status=self.status)
+
+    def launches_per_step(self):
+        # allocate (1) + verify: streaming + decide/sample (2) + commit (1 for B <= 256, else 2)
+        return 1 + 2 + (1 if self.wl.B <= 256 else 2)
+
+
+def algorithmic_bytes(wl, acc):
+    """Bytes the method must move once per step (Section 4.2 verifies every
+    retained position in one pass): every logits row, the q row at each
+    rejection, the q(z)/l(z) gathers, the committed hidden rows read and
+    written, and the small per-request arrays."""
+    B, K, V, H = wl.B, wl.K, wl.V, wl.H
+    esize = 2 if wl.dtype == "bf16" else 4
+    logits = B * (K + 1) * V * esize
+    rejected = int(np.sum(acc < K))
+    q_rows = rejected * V * esize if wl.q is not None else 0
+    gathers = B * K * 2 * 32
+    committed = int(np.sum(acc + 1))
+    commit = 2 * committed * H * 2 if wl.hidden is not None else 0
+    small = B * (K * 4 + K * 4 + 8 * 3 + (K + 1) * 4 * 2 + 4 * 4)
+    return dict(logits=logits, q_rows=q_rows, gathers=gathers, commit=commit, small=small,
+                total=logits + q_rows + gathers + commit + small)
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for name in ("verify.cu", "spec_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2607_25852_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload):
+    """DRAM bytes per launch of the streaming kernel from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "stream_rows_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    entry = rec.get(workload)
+    if not entry or entry.get("source_hash") != kernel_source_hash():
+        return None
+    return entry.get("dram_bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timings (test infrastructure, timed as a reported baseline)
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, seconds, step_repeats=None):
+    """Run the CPU oracle over full batches of the same workload on all host
+    cores (one request per task) until `seconds` of wall time have passed."""
+    import oracle
+    import torch
+    lg = wl.logits.detach().cpu()
+    logits = lg.view(torch.int16).numpy().view(np.uint16) if lg.dtype == torch.bfloat16 else lg.numpy()
+    q = None
+    if wl.q is not None:
+        qc = wl.q.detach().cpu()
+        q = qc.view(torch.int16).numpy().view(np.uint16) if qc.dtype == torch.bfloat16 else qc.numpy()
+    drafts = wl.drafts.cpu().numpy()
+    seeds = wl.seeds.cpu().numpy().view(np.uint64)
+    reqs = wl.request_ids.cpu().numpy().view(np.uint64)
+    pos = wl.pos_base.cpu().numpy()
+    B, K = wl.B, wl.K
+    oracle.load()
+    threads = os.cpu_count() or 1
+
+    def one(i):
+        return oracle.verify_batch(logits, drafts, q, wl.temperature, seeds, reqs, pos, requests=[i])
+
+    rows = 0
+    batches = 0
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        while True:
+            list(ex.map(one, range(B)))
+            rows += B * (K + 1)
+            batches += 1
+            el = time.perf_counter() - t0
+            if (step_repeats is None and el >= seconds) or (step_repeats is not None and batches >= step_repeats):
+                break
+    el = time.perf_counter() - t0
+    return rows, el, threads, batches
+
+
+# ---------------------------------------------------------------------------
+# arms
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    """The reference arm: the CPU oracle, timed on the host cores."""
+    world, rank, local = dist_info()
+    if rank != 0:
+        return 0
+    import torch
+    wl = make_inputs(args, 0, "cpu")
+    R = wl.rows
+    # bounded sample per step: one full batch (all B requests) through the oracle
+    if args.warmup:
+        oracle_sample(wl, 0, step_repeats=1)
+    times = []
+    threads = os.cpu_count() or 1
+    for _ in range(args.steps):
+        rows, el, threads, _ = oracle_sample(wl, 0, step_repeats=1)
+        times.append(el)
+    total = sum(times)
+    value = R * args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"{wl.name}: B={wl.B} K={wl.K} V={wl.V} {wl.dtype} logits, "
+                               f"t={wl.temperature}, q {'bf16' if wl.q is not None else 'one-hot'}",
+                   "sample": "one full batch per step (verification of every request)"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"full batch of {wl.B} requests x {wl.K + 1} rows per step"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    world, rank, local = dist_info()
+    if not torch.cuda.is_available():
+        print(json.dumps({"error": "no CUDA device"}))
+        return 1
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    dist = dist_init(world, "nccl")
+    import paper_2607_25852_gb300 as spec
+
+    wl = make_inputs(args, rank, device)
+    R = wl.rows
+    step = Step(wl, device)
+    stream = torch.cuda.current_stream()
+
+    for _ in range(max(args.warmup, 3)):
+        step.run()
+    torch.cuda.synchronize()
+    assert int(step.status.item()) == 0, "device reported an input error"
+    assert int(step.chosen.item()) == R, "the flat cost table should select the full block"
+    acc = step.acc.cpu().numpy()
+    alg = algorithmic_bytes(wl, acc)
+
+    # ---- device-timed region ----
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    for pair in ev + kev:          # torch creates the CUDA events lazily, at first record
+        for e in pair:
+            e.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            spec.spec_profile_stream_pass(kev[k][0], kev[k][1])
+            step.run()
+            ev[k][1].record(stream)
+        stop.record(stream)
+        torch.cuda.synchronize()
+    barrier(dist)
+    total_ms = start.elapsed_time(stop)
+    total_ms = max_over_ranks(dist, total_ms, device)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    kern_ms = [a.elapsed_time(b) for a, b in kev]
+    ms_per_step = total_ms / args.steps
+    value = world * R * args.steps / (total_ms * 1e-3)
+
+    # ---- end to end through the same API with pinned host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        host = {k: getattr(wl, k).cpu().pin_memory() for k in
+                ("conf", "logits", "drafts", "q", "seeds", "request_ids", "pos_base", "last_tokens",
+                 "hidden") if getattr(wl, k) is not None}
+        dev_in = {k: torch.empty_like(v, device=device) for k, v in host.items()}
+        dev_in.setdefault("q", None)
+        outs_host = [torch.empty_like(t, device="cpu").pin_memory() for t in (step.acc, step.tok, step.ctok, step.coff)]
+        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        d2h = sum(t.numel() * t.element_size() for t in outs_host)
+
+        def e2e_step():
+            for k, v in host.items():
+                dev_in[k].copy_(v, non_blocking=True)
+            step.run(dev_in)
+            for o, d in zip(outs_host, (step.acc, step.tok, step.ctok, step.coff)):
+                o.copy_(d, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        n_e2e = max(3, min(args.steps, 10))
+        barrier(dist)
+        t0 = time.perf_counter()
+        for _ in range(n_e2e):
+            e2e_step()
+        torch.cuda.synchronize()
+        el = max_over_ranks(dist, time.perf_counter() - t0, device)
+        e2e = {"value": world * R * n_e2e / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": n_e2e, "ms_per_step": 1e3 * el / n_e2e}
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+
+    peak, peak_kind = measured_peak()
+    k_ms = statistics.mean(kern_ms)
+    achieved = alg["logits"] / (k_ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
+                "kernel": "stream_rows_kernel", "peak_kind": peak_kind,
+                "algorithmic_bytes_per_launch": alg["logits"], "avg_launch_us": round(1e3 * k_ms, 2),
+                "frac_of_8000": round(achieved / 8000.0, 4)}
+    step_gbs = alg["total"] / (ms_per_step * 1e-3) / 1e9
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        rows, el, threads, batches = oracle_sample(wl, args.cpu_seconds)
+        cpu = {"value": rows / el, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"{batches} full batch(es) of the same workload ({wl.B} requests x "
+                         f"{wl.K + 1} rows), {el:.1f} s wall on {threads} host threads"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": f"{wl.name}: B={wl.B} K={wl.K} V={wl.V} {wl.dtype} logits, "
+                               f"t={wl.temperature}, q {'bf16 [B,K,V]' if wl.q is not None else 'one-hot'}, "
+                               f"H={wl.H}; D-cut ratios 1/4..1 with a flat cost table (T*={R})",
+                   "rows_per_step": R, "l2": "inputs larger than L2 (437.6 MB logits per step)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "roofline": roofline,
+        "step_hbm_gbs": round(step_gbs, 1),
+        "step_frac_of_measured": round(step_gbs / peak, 4),
+        "step_frac_of_8000": round(step_gbs / 8000.0, 4),
+        "algorithmic_bytes_per_step": alg,
+        "step_ms_p10_p50_p90": [float(np.percentile(step_ms, p)) for p in (10, 50, 90)],
+        "mean_accepted": float(acc.mean()),
+        "clocks": clocks.summary(),
+        "e2e": e2e,
+        "gpu_launches": step.launches_per_step() * args.steps,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
