@@ -61,7 +61,9 @@ typedef enum {
   SPEC_ERR_WORKSPACE = 2,   /* workspace missing, too small or misaligned */
   SPEC_ERR_CUDA = 3,        /* a CUDA runtime call failed (e.g. launch) */
   SPEC_ERR_BAD_INPUT = 4,   /* device-detected data error (via *status) */
-  SPEC_ERR_TIMEOUT = 5      /* a bounded device wait gave up (via *status) */
+  SPEC_ERR_TIMEOUT = 5,     /* a bounded device wait gave up (via *status) */
+  SPEC_ERR_TOO_LARGE = 6    /* shape needs more than the static scratch of
+                               spec_verify_static; nothing launched */
 } spec_err;
 
 typedef enum { SPEC_BF16 = 0, SPEC_F32 = 1 } spec_dtype;
@@ -189,6 +191,39 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
                 const int64_t* pos_base, int32_t* accepted_len_out,
                 int32_t* out_tokens, float* p_draft_out, float* row_stats_out,
                 int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * spec_verify_static -- spec_verify for callers that cannot allocate device
+ * memory.  The paper has no counterpart: this is a deployment convenience.
+ * Who needs it: code inside an inference engine that owns all device memory
+ * through its own pool and forbids allocations outside it (under a tight
+ * budget such an allocation may fail, and it escapes the engine's memory
+ * accounting), and code on a latency-critical path that may not call
+ * cudaMalloc, which can synchronise the device.
+ * Same arguments and results as spec_verify, without ws / ws_bytes: the
+ * scratch is a fixed device array of SPEC_STATIC_SCRATCH_BYTES owned by the
+ * library, reserved on every GPU that loads it and held until process exit.
+ *   - Returns SPEC_ERR_TOO_LARGE, launching nothing, when
+ *     spec_verify_workspace(B, K, V) exceeds SPEC_STATIC_SCRATCH_BYTES
+ *     (4 MiB holds about 260,000 16-byte row-chunk partials; B=64, K=16,
+ *     V=201088 needs 86 KB).
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before
+ *     any stream capture.
+ *   - Every call on a device shares the one array, which keeps the previous
+ *     call's contents; each call clears the part that must start at zero.
+ *     Calls that overlap on the GPU (concurrent streams, or several host
+ *     threads) race on the array and give wrong results: serialise them.
+ *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ * ---------------------------------------------------------------------- */
+#define SPEC_STATIC_SCRATCH_BYTES (4u << 20)
+int spec_verify_static(const void* logits, int logits_dtype, const int32_t* row_offsets,
+                       const int32_t* depth, const int32_t* draft_tokens, const void* q,
+                       int q_dtype, int B, int K, int V, float temperature,
+                       const uint64_t* seeds, const uint64_t* request_ids,
+                       const int64_t* pos_base, int32_t* accepted_len_out,
+                       int32_t* out_tokens, float* p_draft_out, float* row_stats_out,
+                       int32_t* status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * spec_commit -- pack the committed round for the drafter's next step

@@ -24,6 +24,7 @@ ERR_WORKSPACE = 2
 ERR_CUDA = 3
 ERR_BAD_INPUT = 4
 ERR_TIMEOUT = 5
+ERR_TOO_LARGE = 6
 
 MAX_DRAFTS = 255
 MAX_ALLOC_POSITIONS = 8192
@@ -32,7 +33,7 @@ MAX_CANDIDATES = 64
 __all__ = [
     "SpecError", "spec_version", "spec_error_string", "spec_budget_from_ratios",
     "spec_allocate_workspace", "spec_allocate", "spec_verify_workspace", "spec_verify",
-    "spec_commit", "spec_profile_stream_pass", "verify_workspace", "library",
+    "spec_verify_static", "spec_commit", "spec_profile_stream_pass", "verify_workspace", "library",
 ]
 
 
@@ -139,6 +140,19 @@ def spec_verify(logits, draft_tokens, q, B, K, V, temperature, seeds, request_id
         _ptr(row_stats_out), _ptr(status), _ptr(ws), ws.numel() * ws.element_size(),
         _stream(stream))
     _check(code, "spec_verify")
+
+
+def spec_verify_static(logits, draft_tokens, q, B, K, V, temperature, seeds, request_ids,
+                       pos_base, accepted_len_out, out_tokens, row_offsets=None, depth=None,
+                       p_draft_out=None, row_stats_out=None, status=None, stream=None):
+    """spec_verify without a workspace argument, for callers that may not
+    allocate device memory (the scratch is a static array of the library)."""
+    code = library().spec_verify_static(
+        _ptr(logits), _dtype(logits), _ptr(row_offsets), _ptr(depth), _ptr(draft_tokens),
+        _ptr(q), _dtype(q), B, K, V, float(temperature), _ptr(seeds), _ptr(request_ids),
+        _ptr(pos_base), _ptr(accepted_len_out), _ptr(out_tokens), _ptr(p_draft_out),
+        _ptr(row_stats_out), _ptr(status), _stream(stream))
+    _check(code, "spec_verify_static")
 
 
 def spec_commit(accepted_len, out_tokens, hidden, B, K, packed_tokens_out, commit_offsets_out,

@@ -23,6 +23,8 @@ SIGNATURES = {
     "spec_verify_workspace": (_SZ, [_I, _I, _I]),
     "spec_verify": (_I, [_P, _I, _P, _P, _P, _P, _I, _I, _I, _I, ctypes.c_float, _P, _P, _P,
                          _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "spec_verify_static": (_I, [_P, _I, _P, _P, _P, _P, _I, _I, _I, _I, ctypes.c_float, _P, _P,
+                                _P, _P, _P, _P, _P, _P, _P]),
     "spec_commit": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
     "spec_profile_stream_pass": (_I, [_P, _P]),
 }

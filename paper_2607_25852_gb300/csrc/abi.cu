@@ -45,6 +45,7 @@ const char* spec_error_string(int code) {
     case SPEC_ERR_CUDA: return "CUDA runtime error";
     case SPEC_ERR_BAD_INPUT: return "bad input data detected on the device";
     case SPEC_ERR_TIMEOUT: return "bounded device wait timed out";
+    case SPEC_ERR_TOO_LARGE: return "shape needs more scratch than the static buffer holds";
     default: return "unknown error code";
   }
 }
