@@ -6,10 +6,15 @@
 //   bits(s_{i,k}) << 32 | (0xFFFF - k) << 16 | (0xFFFF - i)
 // whose descending order is the allocator's total order: s >= 0, so the fp32
 // bit pattern is monotone in s; then shallower k first (the paper's tie rule);
-// then lower request index.  A bitonic network sorts the keys descending; an
-// inclusive scan of floor(s * 2^40) over the sorted order gives every
-// candidate's utility U(T) = prefix[T - 1] exactly, the first maximiser of
-// U / cost is chosen, and the kept prefixes are packed densely.
+// then lower request index.  Keys are unique.
+//
+// Because s_{i,k} is non-increasing in k, each request's K+1 keys already form
+// a run sorted in descending order.  A merge tree of ceil(log2 B) levels sorts
+// the B runs: at every level each key finds its place in the merged pair by
+// one binary search in the partner run.  An inclusive scan of floor(s * 2^40)
+// in sorted order then gives every candidate's utility U(T) = prefix[T - 1]
+// exactly; the first maximiser of U / cost is chosen and the kept prefixes
+// are packed densely.
 #include <float.h>
 #include <math.h>
 
@@ -51,96 +56,147 @@ __device__ __forceinline__ long long block_inclusive_scan(long long x, long long
   return x + before;
 }
 
+// Shared-memory layout (dynamic): two key buffers of N entries, then the
+// confidences [B*K] fp32, then the draft tokens [B*K] int32, then
+// last_tokens [B] int32 and pos_base [B] int64.
+struct AllocSmem {
+  unsigned long long* keys[2];
+  float* conf;
+  int32_t* drafts;
+  int32_t* last;
+  long long* pos;
+};
+
+__device__ __forceinline__ AllocSmem carve(unsigned char* base, int N, int BK, int B) {
+  AllocSmem s;
+  s.keys[0] = reinterpret_cast<unsigned long long*>(base);
+  s.keys[1] = s.keys[0] + N;
+  unsigned char* p = reinterpret_cast<unsigned char*>(s.keys[1] + N);
+  s.pos = reinterpret_cast<long long*>(p);
+  p += (size_t)B * 8;
+  s.conf = reinterpret_cast<float*>(p);
+  p += (size_t)BK * 4;
+  s.drafts = reinterpret_cast<int32_t*>(p);
+  p += (size_t)BK * 4;
+  s.last = reinterpret_cast<int32_t*>(p);
+  return s;
+}
+
+size_t allocate_smem_bytes(int B, int K) {
+  const size_t N = (size_t)B * (K + 1), BK = (size_t)B * K;
+  return N * 16 + (size_t)B * 8 + BK * 8 + (size_t)B * 4 + 16;
+}
+
 __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaunch p) {
-  extern __shared__ unsigned long long smem[];
-  unsigned long long* keys = smem;                                     // [npad]
-  long long* prefix = reinterpret_cast<long long*>(smem + p.npad);     // [npad], later counts
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int B = p.B, K = p.K, N = B * (K + 1), BK = B * K, L0 = K + 1;
+  const AllocSmem sm = carve(smem_raw, N, BK, B);
   __shared__ long long warp_tot[32];
   __shared__ int sh_best_c;
   __shared__ int sh_bad;
-
-  const int B = p.B, K = p.K, N = B * (K + 1), npad = p.npad;
   const int tid = threadIdx.x;
   if (tid == 0) sh_bad = 0;
+
+  // ---- every global input in one round trip, coalesced ----
+  for (int q = tid; q < BK; q += kAllocThreads) {
+    sm.conf[q] = p.conf[q];
+    sm.drafts[q] = p.drafts[q];
+  }
+  for (int i = tid; i < B; i += kAllocThreads) {
+    sm.last[i] = p.last_tokens[i];
+    sm.pos[i] = p.pos_base[i];
+  }
   __syncthreads();
 
-  // ---- Eq. (dcut-score): fp32 prefix products, one request per thread ----
+  // ---- Eq. (dcut-score): fp32 prefix products; run i holds request i ----
   for (int i = tid; i < B; i += kAllocThreads) {
     float s = 1.0f;
-    keys[i * (K + 1)] = position_key(s, 0, i);
+    sm.keys[0][i * L0] = position_key(s, 0, i);
     for (int k = 1; k <= K; ++k) {
-      float c = p.conf[(size_t)i * K + (k - 1)];
+      float c = sm.conf[i * K + (k - 1)];
       if (!(c >= 0.0f && c <= 1.0f)) {
         sh_bad = 1;
         c = 0.0f;
       }
       s = __fmul_rn(s, c);
-      keys[i * (K + 1) + k] = position_key(s, k, i);
+      sm.keys[0][i * L0 + k] = position_key(s, k, i);
     }
   }
-  for (int q = N + tid; q < npad; q += kAllocThreads) keys[q] = 0ull;  // sorts last
   __syncthreads();
 
-  // ---- bitonic sort, descending ----
-  for (int size = 2; size <= npad; size <<= 1) {
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      for (int t = tid; t < (npad >> 1); t += kAllocThreads) {
-        const int lo = 2 * stride * (t / stride) + (t % stride);
-        const int hi = lo + stride;
-        const bool desc = (lo & size) == 0;
-        const unsigned long long a = keys[lo], b = keys[hi];
-        if ((a < b) == desc) {
-          keys[lo] = b;
-          keys[hi] = a;
-        }
+  // ---- merge tree over the B sorted runs (descending) ----
+  int cur = 0;
+  for (long long L = L0; L < N; L *= 2) {
+    const unsigned long long* in = sm.keys[cur];
+    unsigned long long* out = sm.keys[cur ^ 1];
+    for (int e = tid; e < N; e += kAllocThreads) {
+      const long long run = e / L;
+      const long long start = run * L;
+      const long long partner = run ^ 1;
+      const long long pstart = partner * L;
+      const unsigned long long x = in[e];
+      if (pstart >= N) {  // unpaired last run: copied through
+        out[e] = x;
+        continue;
       }
-      __syncthreads();
+      const long long plen = min((long long)N, pstart + L) - pstart;
+      // number of partner keys greater than x (the partner run is descending)
+      int lo = 0, hi = (int)plen;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (in[pstart + mid] > x) lo = mid + 1;
+        else hi = mid;
+      }
+      const long long base = min(start, pstart);
+      out[base + (e - start) + lo] = x;
     }
+    __syncthreads();
+    cur ^= 1;
   }
+  const unsigned long long* keys = sm.keys[cur];
+  long long* prefix = reinterpret_cast<long long*>(sm.keys[cur ^ 1]);  // free buffer
 
   // ---- inclusive scan of floor(s * 2^40) in sorted order ----
-  const int per = (npad + kAllocThreads - 1) / kAllocThreads;
+  const int per = (N + kAllocThreads - 1) / kAllocThreads;
   const int q0 = tid * per;
   long long local = 0;
-  for (int q = q0; q < q0 + per && q < npad; ++q) {
-    const float s = __uint_as_float((unsigned)(keys[q] >> 32));
-    local += q < N ? (long long)__float2ll_rd(s * 0x1p40f) : 0ll;
-  }
+  for (int q = q0; q < q0 + per && q < N; ++q)
+    local += (long long)__float2ll_rd(__uint_as_float((unsigned)(keys[q] >> 32)) * 0x1p40f);
   const long long incl = block_inclusive_scan(local, warp_tot);
   long long run = incl - local;
-  for (int q = q0; q < q0 + per && q < npad; ++q) {
-    const float s = __uint_as_float((unsigned)(keys[q] >> 32));
-    run += q < N ? (long long)__float2ll_rd(s * 0x1p40f) : 0ll;
+  for (int q = q0; q < q0 + per && q < N; ++q) {
+    run += (long long)__float2ll_rd(__uint_as_float((unsigned)(keys[q] >> 32)) * 0x1p40f);
     prefix[q] = run;
   }
   __syncthreads();
 
   // ---- Eq. (dcut-select): first maximiser of U / cost ----
-  if (tid == 0) {
-    int best_c = 0;
-    double best_obj = -INFINITY;
-    for (int c = 0; c < p.M; ++c) {
-      const double util = ldexp((double)prefix[p.cand_T[c] - 1], -40);
-      if (p.utility_out) p.utility_out[c] = util;
-      const double obj = util / p.cand_cost[c];
-      if (obj > best_obj) {
-        best_obj = obj;
-        best_c = c;
+  if (tid < 32) {
+    // utilities in parallel, argmax by lane 0 in candidate order
+    for (int c = tid; c < p.M; c += 32)
+      if (p.utility_out) p.utility_out[c] = ldexp((double)prefix[p.cand_T[c] - 1], -40);
+    if (tid == 0) {
+      int best_c = 0;
+      double best_obj = -INFINITY;
+      for (int c = 0; c < p.M; ++c) {
+        const double obj = ldexp((double)prefix[p.cand_T[c] - 1], -40) / p.cand_cost[c];
+        if (obj > best_obj) {
+          best_obj = obj;
+          best_c = c;
+        }
       }
+      sh_best_c = best_c;
     }
-    sh_best_c = best_c;
   }
   __syncthreads();
   const int T = p.cand_T[sh_best_c];
 
   // ---- keep depths: count the selected positions per request ----
   int* counts = reinterpret_cast<int*>(prefix);  // prefix no longer needed
+  int* offsets = counts + B;                       // [B]
   for (int i = tid; i < B; i += kAllocThreads) counts[i] = 0;
   __syncthreads();
-  for (int q = tid; q < T; q += kAllocThreads) {
-    const int i = 0xFFFF - (int)(keys[q] & 0xFFFFull);
-    atomicAdd(&counts[i], 1);
-  }
+  for (int q = tid; q < T; q += kAllocThreads) atomicAdd(&counts[0xFFFF - (int)(keys[q] & 0xFFFFull)], 1);
   __syncthreads();
 
   // ---- row offsets: exclusive scan of (n_i + 1) = counts ----
@@ -150,7 +206,6 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
   for (int i = b0; i < b0 + perB && i < B; ++i) lsum += counts[i];
   const long long bincl = block_inclusive_scan(lsum, warp_tot);
   long long off = bincl - lsum;
-  int* offsets = reinterpret_cast<int*>(prefix) + B;  // [B+1] after counts
   for (int i = b0; i < b0 + perB && i < B; ++i) {
     offsets[i] = (int)off;
     p.row_offsets_out[i] = (int)off;
@@ -170,8 +225,8 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
       const int i = 0xFFFF - (int)(key & 0xFFFFull);
       const int k = 0xFFFF - (int)((key >> 16) & 0xFFFFull);
       const int row = offsets[i] + k;
-      p.packed_tokens_out[row] = k == 0 ? p.last_tokens[i] : p.drafts[(size_t)i * K + (k - 1)];
-      p.packed_pos_out[row] = p.pos_base[i] + k;
+      p.packed_tokens_out[row] = k == 0 ? sm.last[i] : sm.drafts[i * K + (k - 1)];
+      p.packed_pos_out[row] = sm.pos[i] + k;
     } else {
       p.packed_tokens_out[q] = -1;
       p.packed_pos_out[q] = -1;
@@ -181,10 +236,7 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
 }
 
 cudaError_t launch_allocate(const AllocLaunch& p, cudaStream_t stream) {
-  // keys [npad] u64, then one region reused for the prefix sums [npad] i64 and
-  // for counts [B] + offsets [B+1] i32
-  const size_t region = std::max((size_t)p.npad * 8, ((size_t)2 * p.B + 2) * 4);
-  const size_t smem = (size_t)p.npad * 8 + ((region + 15) / 16) * 16;
+  const size_t smem = allocate_smem_bytes(p.B, p.K);
   cudaError_t err = cudaFuncSetAttribute(allocate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
   if (err != cudaSuccess) return err;

@@ -6,7 +6,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/spec.h"
+#include "spec.h"
 
 namespace spec {
 
