@@ -38,7 +38,8 @@
  * with key = (lo32(seed_i), hi32(seed_i)) and counter =
  *   (lo32(position), lo32(request_id_i), hi32(request_id_i), purpose<<28 | sub)
  *   SPEC_PURPOSE_ACCEPT: sub = 0; u = (word0 >> 8) * 2^-24 in [0, 1)
- *   SPEC_PURPOSE_SAMPLE: sub = v >> 2; E_v = -ln(((word[v & 3] >> 8) + 1) * 2^-24)
+ *   SPEC_PURPOSE_SAMPLE: sub = v >> 2; E_v = -ln((2 * (word[v & 3] >> 9) + 1) * 2^-24),
+ *                        the midpoint of one of 2^23 cells of (0, 1), so E_v > 0
  * so a round replays bit for bit from (seed, request id, position).
  */
 #ifndef SPEC_H_

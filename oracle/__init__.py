@@ -47,6 +47,8 @@ def _declare(lib):
     lib.oracle_accept_uniform.argtypes = [ctypes.c_uint64] * 3
     lib.oracle_accept_uniform.restype = ctypes.c_double
     lib.oracle_race_exponential.argtypes = [ctypes.c_uint64] * 3 + [ctypes.c_uint32]
+    lib.oracle_race_variate.argtypes = [ctypes.c_uint32]
+    lib.oracle_race_variate.restype = ctypes.c_double
     lib.oracle_race_exponential.restype = ctypes.c_double
     lib.oracle_row_stats.argtypes = [_P, ctypes.c_int, ctypes.c_int, ctypes.c_double,
                                      _P, _P, _P]
@@ -107,6 +109,11 @@ def philox4x32_10(ctr, key):
 
 def accept_uniform(seed: int, request: int, position: int) -> float:
     return load().oracle_accept_uniform(seed, request, position)
+
+
+def race_variate(word: int) -> float:
+    """Unit exponential variate of one Philox output word."""
+    return load().oracle_race_variate(word)
 
 
 def race_exponential(seed: int, request: int, position: int, v: int) -> float:

@@ -40,7 +40,9 @@
  *   counter = (lo32(position), lo32(request), hi32(request), purpose<<28 | sub)
  *   purpose ACCEPT = 1 (sub = 0, word 0 used), SAMPLE = 2 (sub = v / 4,
  *   word v % 4 used).  Acceptance uniform: (x >> 8) * 2^-24.  Race variate:
- *   E = -ln(((x >> 8) + 1) * 2^-24).
+ *   E = -ln((2 * (x >> 9) + 1) * 2^-24), the midpoint of one of 2^23 equal
+ *   cells of (0, 1), so that E > 0: a variate of exactly 0 would make its entry
+ *   win whatever its weight, and the draw would no longer follow w / sum(w).
  *
  * Build: gcc -O2 -ffp-contract=off -fPIC -shared (see oracle/build.py).
  * -ffp-contract=off keeps results identical on x86-64 and aarch64.
@@ -130,13 +132,19 @@ double oracle_accept_uniform(uint64_t seed, uint64_t request,
   return (double)(w[0] >> 8) * ldexp(1.0, -24);
 }
 
+/* Unit exponential variate of one Philox word: the word's top 23 bits pick a
+ * cell of (0, 1) and u is that cell's midpoint, so 0 < u < 1 and E > 0. */
+double oracle_race_variate(uint32_t word) {
+  double u = (double)(2u * (word >> 9) + 1u) * ldexp(1.0, -24);
+  return -log(u);
+}
+
 /* Exponential variate E_v of the sampling race at `position`, entry v. */
 double oracle_race_exponential(uint64_t seed, uint64_t request,
                                uint64_t position, uint32_t v) {
   uint32_t w[4];
   draw_words(seed, request, position, OR_PURPOSE_SAMPLE, v >> 2, w);
-  double u = (double)((w[v & 3u] >> 8) + 1u) * ldexp(1.0, -24);
-  return -log(u);
+  return oracle_race_variate(w[v & 3u]);
 }
 
 /* ------------------------------------------------------------------------ */

@@ -78,8 +78,7 @@ def test_variates_follow_the_counter_layout():
         for v in [0, 1, 2, 3, 4, 4097, 201087]:
             w = oracle.philox4x32_10([_u32(pos), _u32(req), _u32(req >> 32), (2 << 28) | (v >> 2)],
                                      [_u32(seed), _u32(seed >> 32)])
-            u = ((int(w[v & 3]) >> 8) + 1) / 2.0**24
-            assert oracle.race_exponential(seed, req, pos, v) == pytest.approx(-np.log(u), rel=1e-15)
+            assert oracle.race_exponential(seed, req, pos, v) == oracle.race_variate(int(w[v & 3]))
 
 
 def test_accept_uniform_is_uniform():
@@ -100,6 +99,32 @@ def test_race_exponentials_are_unit_exponential():
     blocks = e.reshape(-1, 4)
     c = np.corrcoef(blocks.T)
     assert np.max(np.abs(c - np.eye(4))) < 5.0 / np.sqrt(len(blocks))
+
+
+def test_race_variate_is_a_positive_unit_exponential():
+    """Pins of the word -> E map against Exp(1) itself, not against its formula.
+
+    Every variate is > 0: an entry with E = 0 would win the race whatever its
+    weight, so a vocabulary of V entries would send about V / 2^24 of all
+    draws (1.2 % at V = 201088) to an entry that ignores the distribution.
+    The extremes are the Exp(1) quantiles at the outer cell midpoints, and the
+    map is monotone (a larger word is a larger u).
+    """
+    e_min = oracle.race_variate(0xFFFFFFFF)
+    assert e_min > 0.0
+    assert e_min == pytest.approx(-np.log1p(-2.0**-24), rel=1e-9)   # P(E <= e) = 2^-24
+    assert oracle.race_variate(0) == pytest.approx(24 * np.log(2.0), rel=1e-12)
+    assert oracle.race_variate(511) == oracle.race_variate(0)         # low 9 bits unused
+    assert oracle.race_variate(512) < oracle.race_variate(0)
+    # moments over an even sweep of the 2^23 cells: mean 1, variance 1
+    cells = np.arange(0, 1 << 23, 61)
+    e = np.array([oracle.race_variate(int(c) << 9) for c in cells])
+    assert np.all(np.diff(e) < 0)
+    assert e.mean() == pytest.approx(1.0, abs=2e-3)
+    assert e.var() == pytest.approx(1.0, abs=1e-2)
+    # a two-entry race with weights 1 and 1e-12: the small entry wins with
+    # probability about 1e-12, so no cell may let it win outright
+    assert e_min / 1e-12 > oracle.race_variate(0) / 1.0
 
 
 def test_streams_differ_by_every_key_field():
