@@ -161,12 +161,21 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
   char* base = static_cast<char*>(ws);
   p.row_part = reinterpret_cast<spec::RowPartial*>(base + g.row_part_off);
   p.race_part = reinterpret_cast<spec::RacePartial*>(base + g.race_part_off);
+  p.req_rec = reinterpret_cast<spec::ReqRec*>(base + g.req_rec_off);
   p.counters = reinterpret_cast<uint32_t*>(base + g.counters_off);
+  p.req_count = p.counters + B;
   p.R_max = B * (K + 1);
   p.NC = g.NC;
   p.chunk = g.chunk;
   p.NCS = g.NCS;
   p.chunk_s = g.chunk_s;
+  {
+    // 16-byte loads in the sampling pass: V a multiple of 8 (every chunk
+    // starts on a group of 8) and both row bases 16-byte aligned.
+    const size_t esize = logits_dtype == SPEC_F32 ? 4 : 2, qsize = q_dtype == SPEC_F32 ? 4 : 2;
+    const bool q_ok = p.q == nullptr || (reinterpret_cast<uintptr_t>(p.q) % 16 == 0 && (V * qsize) % 16 == 0);
+    p.vec_s = V % 8 == 0 && reinterpret_cast<uintptr_t>(logits) % 16 == 0 && (V * esize) % 16 == 0 && q_ok;
+  }
   return spec::launch_verify(p, stream, ev_before, ev_after) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 

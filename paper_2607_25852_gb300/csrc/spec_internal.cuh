@@ -99,6 +99,17 @@ struct alignas(16) RowPartial {
   int32_t flags;
 };
 
+// A partial written by another CTA of the same kernel: read at L2 (.cg).
+__device__ __forceinline__ RowPartial load_partial_cg(const RowPartial* ptr) {
+  const uint4 v = __ldcg(reinterpret_cast<const uint4*>(ptr));
+  RowPartial r;
+  r.m = __uint_as_float(v.x);
+  r.s = __uint_as_float(v.y);
+  r.idx = (int32_t)v.z;
+  r.flags = (int32_t)v.w;
+  return r;
+}
+
 // Per (request, vocabulary chunk) partial of the sampling pass: the best key
 // and index of the residual race (weights max(0, p - q)) and of the race on p.
 struct alignas(16) RacePartial {
@@ -106,6 +117,17 @@ struct alignas(16) RacePartial {
   int32_t idx_r;
   float key_p;
   int32_t idx_p;
+};
+
+// Per request, written by its decision for the sampling pass (t > 0).
+struct alignas(16) ReqRec {
+  int32_t a;          // accepted drafts; the sampled row is the request's row a
+  int32_t flags;      // bit0 bad input, bit1 a draft was rejected, bit2 residual against a dense q row
+  int32_t z_excl;     // the rejected draft token with one-hot q (excluded from the race), else -1
+  uint32_t position;  // pos_base + a: the Philox position of the sampled token
+  int64_t srow;       // packed row index of the sampled row
+  float M2;           // fl(max * c2) of the sampled row
+  float invS;         // 1 / S of the sampled row
 };
 
 // ---------------------------------------------------------------------------
@@ -134,12 +156,15 @@ struct VerifyLaunch {
   // workspace carve-up
   RowPartial* row_part;   // [R_max * NC]
   RacePartial* race_part; // [B * NCS]
-  uint32_t* counters;     // [B]
+  ReqRec* req_rec;        // [B]
+  uint32_t* counters;     // [B] sampling-pass arrivals per request
+  uint32_t* req_count;    // [B] streaming-pass arrivals per request
   int R_max;              // B * (K + 1)
   int NC;                 // vocabulary chunks per row, streaming pass
   int chunk;              // elements per chunk (multiple of 8)
   int NCS;                // vocabulary chunks per request, sampling pass
   int chunk_s;            // elements per sampling chunk (multiple of 8)
+  bool vec_s;             // sampling pass may use 16-byte loads
 };
 
 struct AllocLaunch {
@@ -176,7 +201,7 @@ struct CommitLaunch {
 // Workspace geometry (device independent).
 struct VerifyGeometry {
   int NC, chunk, NCS, chunk_s;
-  size_t row_part_off, race_part_off, counters_off, bytes;
+  size_t row_part_off, race_part_off, req_rec_off, counters_off, bytes;  // [counters_off, bytes) starts at zero
 };
 VerifyGeometry verify_geometry(int B, int K, int V);
 

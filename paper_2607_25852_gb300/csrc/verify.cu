@@ -4,24 +4,28 @@
 // the drafted tokens in one pass by rejection sampling; temperature 0 is the
 // longest argmax-matching prefix):
 //
-//   stream_rows_kernel   one CTA per (packed row, vocabulary chunk).  Streams
-//                        the chunk once with 16-byte loads and writes a
-//                        16-byte partial: (max, sum of 2^(l*c2 - fl(max*c2)))
-//                        at t > 0, (max, lowest argmax) at t = 0.  This is the
-//                        HBM-bound pass: every retained logit is read once.
-//   decide_sample_kernel one CTA per (request, vocabulary chunk).  Every CTA of
-//                        a request merges the row partials of that request
-//                        (a few hundred bytes), re-derives the accept/reject
-//                        chain (p_j(z_{j+1}) in fp64 from the merged statistics,
-//                        one Philox draw per draft) and then streams its chunk
-//                        of the single row that is sampled (residual row at
-//                        the first rejection, else the bonus row), running the
-//                        exponential race y = argmin E_v / w_v.  The last CTA
-//                        of the request to finish (atomic arrival counter,
-//                        no spinning) merges the race partials and writes y.
+//   stream_rows_kernel  one CTA per (request, row, vocabulary chunk).  Streams
+//                       its chunk once with 16-byte loads and writes a 16-byte
+//                       partial: (max, sum of 2^(l*c2 - fl(max*c2))) at t > 0,
+//                       (max, lowest argmax) at t = 0.  This is the HBM-bound
+//                       pass: every retained logit is read once.  The last CTA
+//                       of a request to finish (arrival counter, no spinning)
+//                       merges the request's partials and runs its decision
+//                       chain: p_j(z_{j+1}) from the merged statistics and one
+//                       Philox draw per draft, the first rejection, the
+//                       committed prefix, the argmax token at t = 0, and at
+//                       t > 0 a record of what the sampling pass needs.
+//                       Decisions of early requests overlap the streaming of
+//                       later ones.
+//   sample_kernel       t > 0 only: one CTA per (request, vocabulary chunk) of
+//                       the single row that is sampled (the residual row at the
+//                       first rejection, else the bonus row), running the
+//                       exponential race y = argmin E_v / w_v.  The last CTA of
+//                       the request to finish merges the race partials and
+//                       writes y.
 //
-// Nothing in the data path waits on another CTA: cross-CTA combination goes
-// through a kernel boundary (rows) or a last-arrival counter (race).
+// Nothing waits on another CTA: cross-CTA combination goes through arrival
+// counters (the last to arrive does the merge) or the kernel boundary.
 #include <float.h>
 #include <math.h>
 
@@ -58,8 +62,10 @@ VerifyGeometry verify_geometry(int B, int K, int V) {
   g.chunk_s = (int)chunk_s;
   g.row_part_off = 0;
   g.race_part_off = round_up((long long)sizeof(RowPartial) * R_max * nc, 256);
-  g.counters_off = g.race_part_off + round_up((long long)sizeof(RacePartial) * B * ncs, 256);
-  g.bytes = g.counters_off + round_up(sizeof(uint32_t) * (long long)B, 256);
+  g.req_rec_off = g.race_part_off + round_up((long long)sizeof(RacePartial) * B * ncs, 256);
+  // zero region: sampling arrivals [B], then streaming arrivals [B]
+  g.counters_off = g.req_rec_off + round_up((long long)sizeof(ReqRec) * B, 256);
+  g.bytes = g.counters_off + round_up(sizeof(uint32_t) * 2LL * B, 256);
   return g;
 }
 
@@ -104,6 +110,229 @@ __device__ __forceinline__ bool key_better(KeyState a, KeyState b) {
 }
 
 // ---------------------------------------------------------------------------
+// Decision chain (the last streaming CTA of a request)
+// ---------------------------------------------------------------------------
+// Shape of request i as the streaming CTAs see it: every CTA of the request
+// reads the same header, so all agree on n and on the arrival target.  A
+// request whose header is inconsistent streams nothing; its (row 0, chunk 0)
+// CTA alone arrives and reports it.
+struct ReqShape {
+  int n;
+  long long row0;
+  bool valid;
+};
+
+__device__ __forceinline__ ReqShape request_shape(const VerifyLaunch& p, int i) {
+  const int n_in = p.depth ? __ldg(p.depth + i) : p.K;
+  long long off0 = (long long)i * (p.K + 1), off1 = off0 + n_in + 1;
+  if (p.row_offsets) {
+    off0 = __ldg(p.row_offsets + i);
+    off1 = __ldg(p.row_offsets + i + 1);
+  }
+  const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
+  ReqShape s;
+  s.valid = n_in >= 0 && n_in <= p.K && off0 >= 0 && off1 == off0 + n_in + 1 && off1 <= p.R_max &&
+            pos >= 0 && pos + n_in <= 0xFFFFFFFFLL;
+  s.n = s.valid ? n_in : 0;
+  s.row0 = s.valid ? off0 : 0;
+  return s;
+}
+
+// All threads of the CTA.  Merges the chunk partials of rows 0..n, tests
+// every kept draft, writes the committed prefix, and either the argmax token
+// (t = 0) or the record of the row to sample (t > 0).  The arithmetic is fp32:
+// p_j(z) = 2^(l_z*c2 - fl(m*c2)) / S carries a relative error of a few 1e-7,
+// inside the 1e-5 tolerance on probabilities, and an acceptance decision can
+// move only where |u - min(1, p/q)| is of that order.
+template <typename T, bool kGreedy>
+__device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs) {
+  const int K = p.K, V = p.V;
+  const float c2 = p.c2;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __shared__ int sh_bad, sh_first_reject;
+  __shared__ uint32_t sh_pos;
+  __shared__ unsigned long long sh_seed, sh_req;
+  __shared__ float sh_m[kMaxRows];
+  __shared__ float sh_S[kMaxRows];
+  __shared__ int32_t sh_g[kMaxRows];
+  __shared__ int32_t sh_z[kMaxRows];
+  __shared__ float sh_pz[kMaxRows];
+  const int n = rs.n;
+  const long long row0 = rs.row0;
+
+  // ---- round trip 1: seeds and draft tokens ----
+  if (threadIdx.x == 0) {
+    sh_pos = (uint32_t)p.pos_base[i];
+    sh_seed = p.seeds[i];
+    sh_req = p.request_ids[i];
+    sh_bad = rs.valid ? 0 : 1;
+    sh_first_reject = n;
+  }
+  for (int j = threadIdx.x; j < K; j += kStreamThreads) sh_z[j] = p.drafts[(size_t)i * K + j];
+  __syncthreads();
+
+  // ---- round trip 2: the row partials (one warp per row, up to four rows
+  // per warp in flight) and, per draft, the target logit and the draft
+  // probability at the drafted token ----
+  const int jd = threadIdx.x;  // this thread's draft, if jd < n
+  float lz = 0.0f, qz = 1.0f;
+  bool zbad = false;
+  if (rs.valid && jd < n) {
+    const int z = sh_z[jd];
+    if (z < 0 || z >= V) {
+      zbad = true;
+    } else if (!kGreedy) {
+      lz = load_elem(static_cast<const T*>(p.logits) + (size_t)(row0 + jd) * V + z);
+      if (p.q) qz = load_any(p.q, p.q_dtype, ((int64_t)i * K + jd) * (int64_t)V + z);
+    }
+  }
+  if (rs.valid) {
+    constexpr int kWarps = kStreamThreads / 32, kInFlight = 4;
+    for (int jb = warp; jb <= n; jb += kWarps * kInFlight) {
+      RowPartial rp[kInFlight];
+#pragma unroll
+      for (int u = 0; u < kInFlight; ++u) {
+        const int j = jb + u * kWarps;
+        rp[u] = RowPartial{-INFINITY, 0.0f, INT_MAX, 0};
+        if (j <= n && lane < p.NC) rp[u] = load_partial_cg(p.row_part + (size_t)(row0 + j) * p.NC + lane);
+      }
+#pragma unroll
+      for (int u = 0; u < kInFlight; ++u) {
+        const int j = jb + u * kWarps;
+        if (j > n) break;
+        const RowPartial* part = p.row_part + (size_t)(row0 + j) * p.NC;
+        int32_t f = rp[u].flags;
+        if (kGreedy) {
+          ArgState best{-INFINITY, INT_MAX};
+          if (lane < p.NC) best = ArgState{rp[u].m, rp[u].idx};
+          for (int cc = lane + 32; cc < p.NC; cc += 32) {
+            const RowPartial r2 = load_partial_cg(part + cc);
+            f |= r2.flags;
+            ArgState o{r2.m, r2.idx};
+            if (arg_better(o, best)) best = o;
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            ArgState other{__shfl_xor_sync(0xFFFFFFFFu, best.v, o),
+                           __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
+            if (arg_better(other, best)) best = other;
+          }
+          f = __reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
+          if (lane == 0) {
+            sh_m[j] = best.v;
+            sh_g[j] = best.idx;
+            if (f || best.idx == INT_MAX) atomicOr(&sh_bad, 1);
+          }
+        } else {
+          float m = rp[u].m;
+          for (int cc = lane + 32; cc < p.NC; cc += 32) m = fmaxf(m, load_partial_cg(part + cc).m);
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+          const float M2 = m * c2;
+          float S = 0.0f;
+          if (rp[u].m != -INFINITY) S += rp[u].s * exp2f(rp[u].m * c2 - M2);
+          for (int cc = lane + 32; cc < p.NC; cc += 32) {
+            const RowPartial r2 = load_partial_cg(part + cc);
+            f |= r2.flags;
+            if (r2.m != -INFINITY) S += r2.s * exp2f(r2.m * c2 - M2);
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xFFFFFFFFu, S, o);
+          f = __reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
+          if (lane == 0) {
+            sh_m[j] = m;
+            sh_S[j] = S;
+            if (f || !(m > -INFINITY) || !(S > 0.0f) || !isfinite(S)) atomicOr(&sh_bad, 1);
+          }
+        }
+      }
+    }
+  }
+  if (zbad) atomicOr(&sh_bad, 1);
+  __syncthreads();
+
+  // ---- acceptance test of every kept draft (one thread per draft) ----
+  if (!sh_bad && jd < n) {
+    const int z = sh_z[jd];
+    bool reject;
+    if (kGreedy) {
+      reject = z != sh_g[jd];
+      sh_pz[jd] = reject ? 0.0f : 1.0f;
+    } else {
+      // l_z * c2 - fl(m * c2) with one rounding
+      const float pz = exp2f(fmaf(lz, c2, -(sh_m[jd] * c2))) / sh_S[jd];
+      const bool qbad = p.q && (!(qz >= 0.0f) || isinf(qz));
+      float r;
+      if (qz > 0.0f)
+        r = fminf(1.0f, pz / qz);
+      else
+        r = pz > 0.0f ? 1.0f : 0.0f;
+      const uint64_t seed = sh_seed;
+      const uint4 w = philox(draw_counter(sh_pos + (uint32_t)jd, sh_req, SPEC_PURPOSE_ACCEPT, 0u),
+                             (uint32_t)seed, (uint32_t)(seed >> 32));
+      const float u = (float)(w.x >> 8) * 0x1p-24f;  // exact
+      reject = !(u < r);
+      sh_pz[jd] = pz;
+      if (qbad) {
+        atomicOr(&sh_bad, 1);
+        reject = false;
+      }
+    }
+    if (reject) atomicMin(&sh_first_reject, jd);
+  }
+  __syncthreads();
+
+  const bool bad = sh_bad != 0;
+  const int a = bad ? 0 : sh_first_reject;
+  int32_t* tok = p.out_tokens + (size_t)i * (K + 1);
+  if (bad) {
+    if (threadIdx.x == 0) report(p.status, SPEC_ERR_BAD_INPUT);
+    for (int j = threadIdx.x; j <= K; j += kStreamThreads) tok[j] = -1;
+    if (threadIdx.x == 0) p.accepted_len[i] = 0;
+    if (p.p_draft)
+      for (int j = threadIdx.x; j < K; j += kStreamThreads) p.p_draft[(size_t)i * K + j] = 0.0f;
+  } else {
+    for (int j = threadIdx.x; j <= K; j += kStreamThreads) {
+      if (j < a) tok[j] = sh_z[j];
+      else if (j > a) tok[j] = -1;
+    }
+    if (threadIdx.x == 0) p.accepted_len[i] = a;
+    if (p.p_draft)
+      for (int j = threadIdx.x; j < K; j += kStreamThreads) p.p_draft[(size_t)i * K + j] = j < n ? sh_pz[j] : 0.0f;
+    if (p.row_stats) {
+      for (int j = threadIdx.x; j <= n; j += kStreamThreads) {
+        float2 st;
+        if (kGreedy) {
+          st = make_float2(sh_m[j], 0.0f);
+        } else {
+          // ln S relative to the exact max / t: S is kept relative to
+          // fl(m * c2), and fmaf gives m * c2 - fl(m * c2) exactly
+          const float resid = fmaf(sh_m[j], c2, -(sh_m[j] * c2));
+          st = make_float2(sh_m[j] * p.inv_t, (log2f(sh_S[j]) - resid) * 0.69314718055994531f);
+        }
+        reinterpret_cast<float2*>(p.row_stats)[row0 + j] = st;
+      }
+    }
+  }
+  if (threadIdx.x == 0) {
+    if (kGreedy) {
+      if (!bad) tok[a] = sh_g[a];
+    } else {
+      ReqRec rec;
+      rec.a = a;
+      rec.flags = (bad ? 1 : 0) | (a < n ? 2 : 0) | (a < n && p.q != nullptr ? 4 : 0);
+      rec.z_excl = (!bad && a < n) ? sh_z[a] : -1;
+      rec.position = sh_pos + (uint32_t)a;
+      rec.srow = row0 + a;
+      rec.M2 = bad ? 0.0f : sh_m[a] * c2;
+      rec.invS = bad ? 0.0f : 1.0f / sh_S[a];
+      p.req_rec[i] = rec;
+    }
+    p.req_count[i] = 0u;  // leave the workspace zeroed for the next call
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Streaming pass
 // ---------------------------------------------------------------------------
 template <typename T>
@@ -143,473 +372,441 @@ template <typename T, bool kGreedy>
 __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const VerifyLaunch p) {
   using VT = Vec<T>;
   constexpr int VEC = VT::N;
-  const int item = blockIdx.x;
-  const int r = item / p.NC;
-  const int c = item - r * p.NC;
-  int R = p.R_max;
-  if (p.row_offsets) R = min(max(__ldg(p.row_offsets + p.B), 0), p.R_max);
-  if (r >= R) return;
+  const int per_req = (p.K + 1) * p.NC;
+  const int i = blockIdx.x / per_req;
+  const int rem = blockIdx.x - i * per_req;
+  const int j = rem / p.NC;
+  const int c = rem - j * p.NC;
+  const ReqShape rs = request_shape(p, i);
+  if (!(rs.valid ? j <= rs.n : (j == 0 && c == 0))) return;
+  __shared__ int sh_last;
+  if (rs.valid) {
+    const long long r = rs.row0 + j;
+    const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.V;
+    const int v0 = c * p.chunk;
+    const int v1 = min(p.V, v0 + p.chunk);
+    const uintptr_t addr = reinterpret_cast<uintptr_t>(row + v0);
+    const int head = min((int)(((16u - (unsigned)(addr & 15u)) & 15u) / sizeof(T)), v1 - v0);
+    const int body0 = v0 + head;
+    const int nvec = (v1 - body0) / VEC;
+    const int tail0 = body0 + nvec * VEC;
+    const float c2 = p.c2;
 
-  const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.V;
-  const int v0 = c * p.chunk;
-  const int v1 = min(p.V, v0 + p.chunk);
-  const uintptr_t addr = reinterpret_cast<uintptr_t>(row + v0);
-  const int head = min((int)(((16u - (unsigned)(addr & 15u)) & 15u) / sizeof(T)), v1 - v0);
-  const int body0 = v0 + head;
-  const int nvec = (v1 - body0) / VEC;
-  const int tail0 = body0 + nvec * VEC;
-  const float c2 = p.c2;
+    // thread state
+    int32_t flags = 0;
+    ArgState g{-INFINITY, INT_MAX};
+    SoftState st{-INFINITY, 0.0f};
+    float M2 = -INFINITY;  // fl(st.m * c2)
 
-  // thread state
-  int32_t flags = 0;
-  ArgState g{-INFINITY, INT_MAX};
-  SoftState st{-INFINITY, 0.0f};
-  float M2 = -INFINITY;  // fl(st.m * c2)
-
-  auto consume_scalar = [&](int v, float x) {
-    if (x != x) {
-      flags |= 1;
-      return;
-    }
-    if (kGreedy) {
-      if (g.idx == INT_MAX || x > g.v) {
-        g.v = x;
-        g.idx = v;
+    auto consume_scalar = [&](int v, float x) {
+      if (x != x) {
+        flags |= 1;
+        return;
       }
-    } else {
-      if (x == INFINITY) flags |= 1;
-      if (x > st.m) {
-        const float M2n = x * c2;
-        st.s = st.s * exp2f(M2 - M2n);
-        st.m = x;
-        M2 = M2n;
-      }
-      if (st.m != -INFINITY) st.s += ex2_approx(fmaf(x, c2, -M2));
-    }
-  };
-
-  // head: elements before the first 16-byte boundary (lowest indices)
-  if ((int)threadIdx.x < head) consume_scalar(v0 + threadIdx.x, load_elem(row + v0 + threadIdx.x));
-
-  // body: 16-byte vectors, kUnroll vectors in flight per thread
-  const uint4* vp = reinterpret_cast<const uint4*>(row + body0);
-  for (int base = threadIdx.x; base < nvec; base += kStreamThreads * kUnroll) {
-    uint4 w[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int vi = base + u * kStreamThreads;
-      w[u] = vi < nvec ? ldg_stream(vp + vi) : make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad);
-    }
-    float tm = VT::vmax(w[0]);
-#pragma unroll
-    for (int u = 1; u < kUnroll; ++u) tm = fmax_nan(tm, VT::vmax(w[u]));
-    if (tm != tm) {
-      flags |= 1;
-      continue;
-    }
-    if (kGreedy) {
-      if (g.idx == INT_MAX || tm > g.v) {
-        // locate the first element equal to the tile max (index order)
-        int found = INT_MAX;
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-#pragma unroll
-          for (int e = 0; e < VEC; ++e) {
-            if (found == INT_MAX && VT::get(w[u], e) == tm)
-              found = body0 + (base + u * kStreamThreads) * VEC + e;
-          }
-        }
-        g.v = tm;
-        g.idx = found;
-      }
-    } else {
-      if (tm == INFINITY) flags |= 1;
-      if (tm > st.m) {
-        const float M2n = tm * c2;
-        st.s = st.s * exp2f(M2 - M2n);
-        st.m = tm;
-        M2 = M2n;
-      }
-      if (st.m != -INFINITY) {
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-#pragma unroll
-          for (int e = 0; e < VEC; ++e) acc[e & 3] += ex2_approx(fmaf(VT::get(w[u], e), c2, -M2));
-        }
-        st.s += (acc[0] + acc[1]) + (acc[2] + acc[3]);
-      }
-    }
-  }
-
-  // tail: the last < VEC elements (highest indices)
-  if (tail0 + (int)threadIdx.x < v1)
-    consume_scalar(tail0 + threadIdx.x, load_elem(row + tail0 + threadIdx.x));
-
-  // ---- CTA reduction ----
-  __shared__ float sh_a[kStreamThreads / 32];
-  __shared__ float sh_b[kStreamThreads / 32];
-  __shared__ int32_t sh_i[kStreamThreads / 32];
-  __shared__ int32_t sh_f[kStreamThreads / 32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  flags = __reduce_or_sync(0xFFFFFFFFu, (unsigned)flags);
-  if (kGreedy) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      ArgState other{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
-      if (arg_better(other, g)) g = other;
-    }
-    if (lane == 0) {
-      sh_a[warp] = g.v;
-      sh_i[warp] = g.idx;
-      sh_f[warp] = flags;
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      ArgState best{sh_a[0], sh_i[0]};
-      int32_t f = sh_f[0];
-      for (int k = 1; k < kStreamThreads / 32; ++k) {
-        ArgState o{sh_a[k], sh_i[k]};
-        if (arg_better(o, best)) best = o;
-        f |= sh_f[k];
-      }
-      RowPartial out;
-      out.m = best.v;
-      out.s = 0.0f;
-      out.idx = best.idx;
-      out.flags = f;
-      p.row_part[(size_t)r * p.NC + c] = out;
-    }
-  } else {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      SoftState other{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)};
-      st = soft_merge(st, other, c2);
-    }
-    if (lane == 0) {
-      sh_a[warp] = st.m;
-      sh_b[warp] = st.s;
-      sh_f[warp] = flags;
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      SoftState acc{sh_a[0], sh_b[0]};
-      int32_t f = sh_f[0];
-      for (int k = 1; k < kStreamThreads / 32; ++k) {
-        acc = soft_merge(acc, SoftState{sh_a[k], sh_b[k]}, c2);
-        f |= sh_f[k];
-      }
-      RowPartial out;
-      out.m = acc.m;
-      out.s = acc.s;
-      out.idx = 0;
-      out.flags = f;
-      p.row_part[(size_t)r * p.NC + c] = out;
-    }
-  }
-}
-
-// ---------------------------------------------------------------------------
-// Decision chain + sampling pass
-// ---------------------------------------------------------------------------
-// 2^e in double from an exactly known exponent: integer part by scaling, the
-// fractional part through exp2f (relative error ~1e-7).
-__device__ __forceinline__ double exp2_split(double e) {
-  if (e < -1074.0) return 0.0;
-  const double ei = floor(e);
-  const float f = (float)(e - ei);
-  return ldexp((double)exp2f(f), (int)ei);
-}
-
-template <typename T, bool kGreedy>
-__global__ void __launch_bounds__(kSampleThreads) decide_sample_kernel(const VerifyLaunch p) {
-  const int i = blockIdx.x / p.NCS;
-  const int cs = blockIdx.x - i * p.NCS;
-  const int K = p.K, V = p.V;
-  const float c2 = p.c2;
-
-  __shared__ int sh_n, sh_bad, sh_first_reject, sh_last;
-  __shared__ long long sh_row0;
-  __shared__ uint32_t sh_pos;
-  __shared__ float sh_m[kMaxRows];
-  __shared__ double sh_S[kMaxRows];
-  __shared__ int32_t sh_g[kMaxRows];
-  __shared__ float sh_pz[kMaxRows];
-
-  if (threadIdx.x == 0) {
-    int n = p.depth ? p.depth[i] : K;
-    int bad = 0;
-    if (n < 0 || n > K) {
-      bad = 1;
-      n = 0;
-    }
-    long long row0 = (long long)i * (K + 1);
-    if (p.row_offsets) {
-      row0 = p.row_offsets[i];
-      const long long row1 = p.row_offsets[i + 1];
-      if (row0 < 0 || row1 != row0 + n + 1 || row1 > p.R_max) {
-        bad = 1;
-        row0 = 0;
-        n = 0;
-      }
-    }
-    const long long pos = p.pos_base[i];
-    if (pos < 0 || pos + n > 0xFFFFFFFFLL) bad = 1;
-    sh_n = n;
-    sh_row0 = row0;
-    sh_pos = (uint32_t)pos;
-    sh_bad = bad;
-    sh_first_reject = n;
-  }
-  __syncthreads();
-  const int n = sh_n;
-  const long long row0 = sh_row0;
-
-  // ---- merge the streaming partials of rows 0..n (one warp per row) ----
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (!sh_bad) {
-    for (int j = warp; j <= n; j += kSampleThreads / 32) {
-      const RowPartial* part = p.row_part + (size_t)(row0 + j) * p.NC;
-      int32_t f = 0;
       if (kGreedy) {
-        ArgState best{-INFINITY, INT_MAX};
-        for (int cc = lane; cc < p.NC; cc += 32) {
-          const RowPartial rp = part[cc];
-          f |= rp.flags;
-          ArgState o{rp.m, rp.idx};
-          if (arg_better(o, best)) best = o;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          ArgState other{__shfl_xor_sync(0xFFFFFFFFu, best.v, o),
-                         __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
-          if (arg_better(other, best)) best = other;
-        }
-        f = __reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
-        if (lane == 0) {
-          sh_m[j] = best.v;
-          sh_g[j] = best.idx;
-          if (f || best.idx == INT_MAX) atomicOr(&sh_bad, 1);
+        if (g.idx == INT_MAX || x > g.v) {
+          g.v = x;
+          g.idx = v;
         }
       } else {
-        float m = -INFINITY;
-        for (int cc = lane; cc < p.NC; cc += 32) m = fmaxf(m, part[cc].m);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-        const float M2 = m * c2;
-        double S = 0.0;
-        for (int cc = lane; cc < p.NC; cc += 32) {
-          const RowPartial rp = part[cc];
-          f |= rp.flags;
-          if (rp.m != -INFINITY) S += (double)rp.s * (double)exp2f(rp.m * c2 - M2);
+        if (x == INFINITY) flags |= 1;
+        if (x > st.m) {
+          const float M2n = x * c2;
+          st.s = st.s * exp2f(M2 - M2n);
+          st.m = x;
+          M2 = M2n;
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xFFFFFFFFu, S, o);
-        f = __reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
-        if (lane == 0) {
-          sh_m[j] = m;
-          sh_S[j] = S;
-          if (f || !(m > -INFINITY) || !(S > 0.0) || !isfinite(S)) atomicOr(&sh_bad, 1);
-        }
+        if (st.m != -INFINITY) st.s += ex2_approx(fmaf(x, c2, -M2));
       }
-    }
-  }
-  __syncthreads();
+    };
 
-  // ---- acceptance test of every kept draft (one thread per draft) ----
-  const uint64_t seed = p.seeds[i];
-  const uint64_t req = p.request_ids[i];
-  if (!sh_bad) {
-    for (int j = threadIdx.x; j < n; j += kSampleThreads) {
-      const int z = p.drafts[(size_t)i * K + j];
-      if (z < 0 || z >= V) {
-        atomicOr(&sh_bad, 1);
+    // head: elements before the first 16-byte boundary (lowest indices)
+    if ((int)threadIdx.x < head) consume_scalar(v0 + threadIdx.x, load_elem(row + v0 + threadIdx.x));
+
+    // body: 16-byte vectors, kUnroll vectors in flight per thread
+    const uint4* vp = reinterpret_cast<const uint4*>(row + body0);
+    for (int base = threadIdx.x; base < nvec; base += kStreamThreads * kUnroll) {
+      uint4 w[kUnroll];
+  #pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int vi = base + u * kStreamThreads;
+        w[u] = vi < nvec ? ldg_stream(vp + vi) : make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad);
+      }
+      float tm = VT::vmax(w[0]);
+  #pragma unroll
+      for (int u = 1; u < kUnroll; ++u) tm = fmax_nan(tm, VT::vmax(w[u]));
+      if (tm != tm) {
+        flags |= 1;
         continue;
       }
-      bool reject;
       if (kGreedy) {
-        reject = z != sh_g[j];
-        sh_pz[j] = reject ? 0.0f : 1.0f;
-      } else {
-        const float lz = load_elem(static_cast<const T*>(p.logits) + (size_t)(row0 + j) * V + z);
-        const double e = (double)lz * (double)c2 - (double)(sh_m[j] * c2);
-        const double pz = exp2_split(e) / sh_S[j];
-        double qz = 1.0;
-        if (p.q) {
-          qz = (double)load_any(p.q, p.q_dtype, ((int64_t)i * K + j) * (int64_t)V + z);
-          if (!(qz >= 0.0) || isinf(qz)) {
-            atomicOr(&sh_bad, 1);
-            continue;
-          }
-        }
-        double r;
-        if (qz > 0.0)
-          r = fmin(1.0, pz / qz);
-        else
-          r = pz > 0.0 ? 1.0 : 0.0;
-        const uint4 w = philox(draw_counter(sh_pos + (uint32_t)j, req, SPEC_PURPOSE_ACCEPT, 0u),
-                               (uint32_t)seed, (uint32_t)(seed >> 32));
-        const double u = (double)(w.x >> 8) * 0x1p-24;
-        reject = !(u < r);
-        sh_pz[j] = (float)pz;
-      }
-      if (reject) atomicMin(&sh_first_reject, j);
-    }
-  }
-  __syncthreads();
-
-  const bool bad = sh_bad != 0;
-  const int a = bad ? 0 : sh_first_reject;
-  const bool rejected = a < n;
-  int32_t* tok = p.out_tokens + (size_t)i * (K + 1);
-
-  // ---- outputs owned by chunk 0 of the request ----
-  if (cs == 0) {
-    if (bad) {
-      if (threadIdx.x == 0) report(p.status, SPEC_ERR_BAD_INPUT);
-      for (int j = threadIdx.x; j <= K; j += kSampleThreads) tok[j] = -1;
-      if (threadIdx.x == 0) p.accepted_len[i] = 0;
-      if (p.p_draft)
-        for (int j = threadIdx.x; j < K; j += kSampleThreads) p.p_draft[(size_t)i * K + j] = 0.0f;
-    } else {
-      for (int j = threadIdx.x; j <= K; j += kSampleThreads) {
-        if (j < a) tok[j] = p.drafts[(size_t)i * K + j];
-        else if (j > a) tok[j] = -1;
-      }
-      if (threadIdx.x == 0) p.accepted_len[i] = a;
-      if (p.p_draft)
-        for (int j = threadIdx.x; j < K; j += kSampleThreads)
-          p.p_draft[(size_t)i * K + j] = j < n ? sh_pz[j] : 0.0f;
-      if (p.row_stats) {
-        for (int j = threadIdx.x; j <= n; j += kSampleThreads) {
-          float2 rs;
-          if (kGreedy) {
-            rs = make_float2(sh_m[j], 0.0f);
-          } else {
-            // ln S relative to the exact max/t (S is kept relative to fl(max*c2))
-            const double corr = ((double)(sh_m[j] * c2) - (double)sh_m[j] * (double)c2) * 0.6931471805599453;
-            rs = make_float2(sh_m[j] * p.inv_t, (float)(log(sh_S[j]) + corr));
-          }
-          reinterpret_cast<float2*>(p.row_stats)[row0 + j] = rs;
-        }
-      }
-      if (kGreedy && threadIdx.x == 0) tok[a] = sh_g[a];
-    }
-  }
-  if (kGreedy) return;
-
-  // ---- sampling pass over chunk cs of the row to be sampled ----
-  KeyState best_r{INFINITY, INT_MAX};  // residual race (or the bonus race)
-  KeyState best_p{INFINITY, INT_MAX};  // race on p, fallback of an empty residual
-  if (!bad) {
-    const long long srow = row0 + a;
-    const T* row = static_cast<const T*>(p.logits) + (size_t)srow * V;
-    const float M2 = sh_m[a] * c2;
-    const float invS = (float)(1.0 / sh_S[a]);
-    const int z_excl = rejected ? p.drafts[(size_t)i * K + a] : -1;
-    const bool general_q = rejected && p.q != nullptr;
-    const void* qrow = general_q ? (const void*)((const char*)p.q + ((size_t)i * K + a) * (size_t)V *
-                                                                       (p.q_dtype == SPEC_F32 ? 4 : 2))
-                                 : nullptr;
-    const uint32_t position = sh_pos + (uint32_t)a;
-    const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
-    const int v0 = cs * p.chunk_s;
-    const int v1 = min(V, v0 + p.chunk_s);
-    // groups of 4 consecutive entries share one Philox block
-    for (int grp = (v0 >> 2) + threadIdx.x; grp * 4 < v1; grp += kSampleThreads) {
-      const uint4 rnd = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)grp), k0, k1);
-      const uint32_t words[4] = {rnd.x, rnd.y, rnd.z, rnd.w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int v = grp * 4 + e;
-        if (v >= v1) break;
-        const float x = load_elem(row + v);
-        const float ew = ex2_approx(fmaf(x, c2, -M2));  // p_v * S
-        const float d = (float)(0xFFFFFFu - (words[e] >> 8)) * 0x1p-24f;  // 1 - U', exact
-        if (general_q) {
-          const float pv = ew * invS;
-          const float qv = load_any(qrow, p.q_dtype, v);
-          const float wr = fmaxf(0.0f, pv - qv);
-          if (wr > 0.0f && d < best_r.key * wr) {
-            const float key = -log1pf(-d) / wr;
-            if (key < best_r.key) best_r = KeyState{key, v};
-          }
-          if (pv > 0.0f && d < best_p.key * pv) {
-            const float key = -log1pf(-d) / pv;
-            if (key < best_p.key) best_p = KeyState{key, v};
-          }
-        } else {
-          if (ew > 0.0f && d < (v == z_excl ? best_p.key : best_r.key) * ew) {
-            const float key = -log1pf(-d) / ew;
-            if (v == z_excl) {
-              if (key < best_p.key) best_p = KeyState{key, v};
-            } else if (key < best_r.key) {
-              best_r = KeyState{key, v};
+        if (g.idx == INT_MAX || tm > g.v) {
+          // locate the first element equal to the tile max (index order)
+          int found = INT_MAX;
+  #pragma unroll
+          for (int u = 0; u < kUnroll; ++u) {
+  #pragma unroll
+            for (int e = 0; e < VEC; ++e) {
+              if (found == INT_MAX && VT::get(w[u], e) == tm)
+                found = body0 + (base + u * kStreamThreads) * VEC + e;
             }
           }
+          g.v = tm;
+          g.idx = found;
+        }
+      } else {
+        if (tm == INFINITY) flags |= 1;
+        if (tm > st.m) {
+          const float M2n = tm * c2;
+          st.s = st.s * exp2f(M2 - M2n);
+          st.m = tm;
+          M2 = M2n;
+        }
+        if (st.m != -INFINITY) {
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  #pragma unroll
+          for (int u = 0; u < kUnroll; ++u) {
+  #pragma unroll
+            for (int e = 0; e < VEC; ++e) acc[e & 3] += ex2_approx(fmaf(VT::get(w[u], e), c2, -M2));
+          }
+          st.s += (acc[0] + acc[1]) + (acc[2] + acc[3]);
         }
       }
     }
-    if (!general_q) {
-      // the race on p is the residual race plus the excluded draft token
-      if (key_better(best_r, best_p)) best_p = best_r;
+
+    // tail: the last < VEC elements (highest indices)
+    if (tail0 + (int)threadIdx.x < v1)
+      consume_scalar(tail0 + threadIdx.x, load_elem(row + tail0 + threadIdx.x));
+
+    // ---- CTA reduction ----
+    __shared__ float sh_a[kStreamThreads / 32];
+    __shared__ float sh_b[kStreamThreads / 32];
+    __shared__ int32_t sh_i[kStreamThreads / 32];
+    __shared__ int32_t sh_f[kStreamThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    flags = __reduce_or_sync(0xFFFFFFFFu, (unsigned)flags);
+    if (kGreedy) {
+  #pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        ArgState other{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
+        if (arg_better(other, g)) g = other;
+      }
+      if (lane == 0) {
+        sh_a[warp] = g.v;
+        sh_i[warp] = g.idx;
+        sh_f[warp] = flags;
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        ArgState best{sh_a[0], sh_i[0]};
+        int32_t f = sh_f[0];
+        for (int k = 1; k < kStreamThreads / 32; ++k) {
+          ArgState o{sh_a[k], sh_i[k]};
+          if (arg_better(o, best)) best = o;
+          f |= sh_f[k];
+        }
+        RowPartial out;
+        out.m = best.v;
+        out.s = 0.0f;
+        out.idx = best.idx;
+        out.flags = f;
+        p.row_part[(size_t)r * p.NC + c] = out;
+      }
+    } else {
+  #pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        SoftState other{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)};
+        st = soft_merge(st, other, c2);
+      }
+      if (lane == 0) {
+        sh_a[warp] = st.m;
+        sh_b[warp] = st.s;
+        sh_f[warp] = flags;
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        SoftState acc{sh_a[0], sh_b[0]};
+        int32_t f = sh_f[0];
+        for (int k = 1; k < kStreamThreads / 32; ++k) {
+          acc = soft_merge(acc, SoftState{sh_a[k], sh_b[k]}, c2);
+          f |= sh_f[k];
+        }
+        RowPartial out;
+        out.m = acc.m;
+        out.s = acc.s;
+        out.idx = 0;
+        out.flags = f;
+        p.row_part[(size_t)r * p.NC + c] = out;
+      }
     }
   }
+  // ---- arrival; the last CTA of the request decides it ----
+  if (threadIdx.x == 0) {
+    __threadfence();  // the partial above before the count
+    const uint32_t target = rs.valid ? (uint32_t)(rs.n + 1) * (uint32_t)p.NC : 1u;
+    sh_last = atomicAdd(p.req_count + i, 1u) == target - 1u;
+  }
+  __syncthreads();
+  if (!sh_last) return;
+  __threadfence();  // the other CTAs' partials after their counts
+  decide_request<T, kGreedy>(p, i, rs);
+}
 
-  // ---- CTA reduction of the two races ----
-  __shared__ KeyState sh_r[kSampleThreads / 32], sh_p[kSampleThreads / 32];
+// ---------------------------------------------------------------------------
+// Sampling pass (t > 0)
+// ---------------------------------------------------------------------------
+// Eight consecutive entries of a row as floats, from 16-byte loads.
+template <typename T>
+struct Row8;
+template <>
+struct Row8<__nv_bfloat16> {
+  __device__ static void load(const void* row, int g8, float x[8]) {
+    const uint4 w = ldg_stream(static_cast<const uint4*>(row) + g8);
+    x[0] = bf16_lo(w.x);
+    x[1] = bf16_hi(w.x);
+    x[2] = bf16_lo(w.y);
+    x[3] = bf16_hi(w.y);
+    x[4] = bf16_lo(w.z);
+    x[5] = bf16_hi(w.z);
+    x[6] = bf16_lo(w.w);
+    x[7] = bf16_hi(w.w);
+  }
+};
+template <>
+struct Row8<float> {
+  __device__ static void load(const void* row, int g8, float x[8]) {
+    const uint4 a = ldg_stream(static_cast<const uint4*>(row) + 2 * g8);
+    const uint4 b = ldg_stream(static_cast<const uint4*>(row) + 2 * g8 + 1);
+    x[0] = __uint_as_float(a.x);
+    x[1] = __uint_as_float(a.y);
+    x[2] = __uint_as_float(a.z);
+    x[3] = __uint_as_float(a.w);
+    x[4] = __uint_as_float(b.x);
+    x[5] = __uint_as_float(b.y);
+    x[6] = __uint_as_float(b.z);
+    x[7] = __uint_as_float(b.w);
+  }
+};
+
+// Exponential race entries.  The race variate of a Philox word is
+// E = -ln(u), u = (2 * (word >> 9) + 1) * 2^-24; with m = 2^24 * (1 - u), an
+// odd integer below 2^24, E = -ln(1 - m * 2^-24) exactly as in the oracle.
+__device__ __forceinline__ uint32_t race_m(uint32_t word) { return ((word >> 8) & 0xFFFFFEu) ^ 0xFFFFFFu; }
+
+// One entry with weight w: key E / w.  The filter m < thr24 * w, thr24 =
+// 2^24 * (a key some lane of the warp already holds), skips the logarithm
+// when the entry cannot win (E >= 1 - u); a weight of 0 never passes it.
+// Entries arrive in increasing v per thread, so the strict comparison keeps
+// the lowest index on ties.
+__device__ __forceinline__ void race_entry(KeyState& best, float& thr24, float w, uint32_t m, int v) {
+  const float mf = (float)m;
+  if (mf < thr24 * w) {
+    const float key = -log1pf(-(mf * 0x1p-24f)) / w;
+    if (key < best.key) {
+      best = KeyState{key, v};
+      thr24 = fminf(thr24, key * 0x1p24f);
+    }
+  }
+}
+
+// After each group the warp shares its lowest key, so that an entry takes the
+// logarithm only if it could lead the whole warp (otherwise nearly every step
+// has some lane on the slow path).  Keys are >= 0 or +inf, so their bit
+// patterns order like unsigned integers.  Lanes whose chunk ended earlier have
+// left the loop; the reduction runs over the lanes still in it.
+__device__ __forceinline__ float warp_thr24(const KeyState& best) {
+  const unsigned act = __activemask();
+  return __uint_as_float(__reduce_min_sync(act, __float_as_uint(best.key))) * 0x1p24f;
+}
+
+// Race over [v0, v1) of the sampled row.  kGeneral: residual weights
+// max(0, p - q) into best_r.  Otherwise weights p * S (S the row's sum, which
+// does not change the argmin), the excluded draft token z_excl into best_p and
+// every other entry into best_r.
+// Vector form: 16-byte loads, groups of 8 entries (two Philox blocks) per
+// thread and step; needs v0, v1 multiples of 8 and aligned rows.
+template <typename T, typename Q, bool kGeneral>
+__device__ __forceinline__ void race_chunk_vec(const void* row, const void* qrow, int z_excl, int v0, int v1,
+                                               float c2, float M2, float invS, uint32_t position,
+                                               uint64_t req, uint32_t k0, uint32_t k1, KeyState& best_r,
+                                               KeyState& best_p) {
+  float thr24 = best_r.key * 0x1p24f;
+  for (int g8 = (v0 >> 3) + threadIdx.x; g8 * 8 < v1; g8 += kSampleThreads) {
+    float x[8], qv[8];
+    Row8<T>::load(row, g8, x);
+    if (kGeneral) Row8<Q>::load(qrow, g8, qv);
+    const uint4 r0 = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)(2 * g8)), k0, k1);
+    const uint4 r1 = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)(2 * g8 + 1)), k0, k1);
+    const uint32_t words[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int v = g8 * 8 + e;
+      const float ew = ex2_approx(fmaf(x[e], c2, -M2));  // p_v * S
+      const uint32_t m = race_m(words[e]);
+      if (kGeneral) {
+        race_entry(best_r, thr24, fmaxf(0.0f, ew * invS - qv[e]), m, v);
+      } else if (v == z_excl) {
+        float own = best_p.key * 0x1p24f;
+        race_entry(best_p, own, ew, m, v);
+      } else {
+        race_entry(best_r, thr24, ew, m, v);
+      }
+    }
+    thr24 = fminf(thr24, warp_thr24(best_r));
+  }
+}
+
+// Scalar form of the same race (any alignment, any V): groups of 4 entries
+// (one Philox block) per thread and step.
+template <typename T, bool kGeneral>
+__device__ __forceinline__ void race_chunk_scalar(const T* row, const void* qrow, int q_dtype, int z_excl,
+                                                  int v0, int v1, float c2, float M2, float invS,
+                                                  uint32_t position, uint64_t req, uint32_t k0, uint32_t k1,
+                                                  KeyState& best_r, KeyState& best_p) {
+  float thr24 = best_r.key * 0x1p24f;
+  for (int grp = (v0 >> 2) + threadIdx.x; grp * 4 < v1; grp += kSampleThreads) {
+    const uint4 rnd = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)grp), k0, k1);
+    const uint32_t words[4] = {rnd.x, rnd.y, rnd.z, rnd.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int v = grp * 4 + e;
+      if (v < v0 || v >= v1) continue;
+      const float ew = ex2_approx(fmaf(load_elem(row + v), c2, -M2));  // p_v * S
+      const uint32_t m = race_m(words[e]);
+      if (kGeneral) {
+        race_entry(best_r, thr24, fmaxf(0.0f, ew * invS - load_any(qrow, q_dtype, v)), m, v);
+      } else if (v == z_excl) {
+        float own = best_p.key * 0x1p24f;
+        race_entry(best_p, own, ew, m, v);
+      } else {
+        race_entry(best_r, thr24, ew, m, v);
+      }
+    }
+    thr24 = fminf(thr24, warp_thr24(best_r));
+  }
+}
+
+// Minimum key over the CTA (valid in thread 0).  sh: kSampleThreads / 32 slots.
+__device__ __forceinline__ KeyState cta_min_key(KeyState b, KeyState* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    KeyState orr{__shfl_xor_sync(0xFFFFFFFFu, best_r.key, o), __shfl_xor_sync(0xFFFFFFFFu, best_r.idx, o)};
-    KeyState op{__shfl_xor_sync(0xFFFFFFFFu, best_p.key, o), __shfl_xor_sync(0xFFFFFFFFu, best_p.idx, o)};
-    if (key_better(orr, best_r)) best_r = orr;
-    if (key_better(op, best_p)) best_p = op;
+    KeyState other{__shfl_xor_sync(0xFFFFFFFFu, b.key, o), __shfl_xor_sync(0xFFFFFFFFu, b.idx, o)};
+    if (key_better(other, b)) b = other;
   }
-  if (lane == 0) {
-    sh_r[warp] = best_r;
-    sh_p[warp] = best_p;
-  }
+  if (lane == 0) sh[warp] = b;
   __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int k = 1; k < kSampleThreads / 32; ++k) {
-      if (key_better(sh_r[k], sh_r[0])) sh_r[0] = sh_r[k];
-      if (key_better(sh_p[k], sh_p[0])) sh_p[0] = sh_p[k];
+  if (threadIdx.x == 0)
+    for (int k = 0; k < kSampleThreads / 32; ++k)
+      if (key_better(sh[k], b)) b = sh[k];
+  __syncthreads();
+  return b;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyLaunch p) {
+  const int i = blockIdx.x / p.NCS;
+  const int cs = blockIdx.x - i * p.NCS;
+  const int V = p.V;
+  const ReqRec rec = p.req_rec[i];
+  if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
+  const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+  const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
+  __shared__ int sh_last, sh_y;
+  __shared__ KeyState sh_red[kSampleThreads / 32];
+
+  // Residual race at a rejection with a drafter distribution q; otherwise the
+  // race on p (bonus row), or on p without the rejected one-hot draft.
+  const bool general_q = (rec.flags & 4) != 0;
+  const T* row = static_cast<const T*>(p.logits) + (size_t)rec.srow * V;
+  const size_t qsize = p.q_dtype == SPEC_F32 ? 4 : 2;
+  const void* qrow =
+      general_q ? (const void*)((const char*)p.q + ((size_t)i * p.K + rec.a) * (size_t)V * qsize) : nullptr;
+  const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  const float c2 = p.c2;
+  KeyState best_r{INFINITY, INT_MAX};
+  KeyState best_p{INFINITY, INT_MAX};  // one-hot rejection: the excluded draft
+  {
+    const int v0 = cs * p.chunk_s;
+    const int v1 = min(V, v0 + p.chunk_s);
+    if (p.vec_s) {
+      if (general_q) {
+        if (p.q_dtype == SPEC_F32)
+          race_chunk_vec<T, float, true>(row, qrow, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position, req,
+                                         k0, k1, best_r, best_p);
+        else
+          race_chunk_vec<T, __nv_bfloat16, true>(row, qrow, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
+                                                 rec.position, req, k0, k1, best_r, best_p);
+      } else {
+        race_chunk_vec<T, T, false>(row, nullptr, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position, req,
+                                    k0, k1, best_r, best_p);
+      }
+    } else if (general_q) {
+      race_chunk_scalar<T, true>(row, qrow, p.q_dtype, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position,
+                                 req, k0, k1, best_r, best_p);
+    } else {
+      race_chunk_scalar<T, false>(row, nullptr, p.q_dtype, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
+                                  rec.position, req, k0, k1, best_r, best_p);
     }
+    // one-hot: the race on p is the residual race plus the excluded draft
+    if (!general_q && key_better(best_r, best_p)) best_p = best_r;
+  }
+
+  // ---- CTA reduction; the last CTA of the request to arrive merges ----
+  best_r = cta_min_key(best_r, sh_red);
+  best_p = cta_min_key(best_p, sh_red);
+  if (threadIdx.x == 0) {
     RacePartial rp;
-    rp.key_r = sh_r[0].key;
-    rp.idx_r = sh_r[0].idx;
-    rp.key_p = sh_p[0].key;
-    rp.idx_p = sh_p[0].idx;
+    rp.key_r = best_r.key;
+    rp.idx_r = best_r.idx;
+    rp.key_p = best_p.key;
+    rp.idx_p = best_p.idx;
     p.race_part[(size_t)i * p.NCS + cs] = rp;
     __threadfence();
-    const uint32_t prev = atomicAdd(p.counters + i, 1u);
-    sh_last = prev == (uint32_t)(p.NCS - 1);
+    sh_last = atomicAdd(p.counters + i, 1u) == (uint32_t)(p.NCS - 1);
   }
   __syncthreads();
-  if (!sh_last || threadIdx.x != 0) return;
+  if (!sh_last) return;
 
-  // ---- last CTA of the request: merge the race partials, write y ----
   __threadfence();
-  KeyState r_all{INFINITY, INT_MAX}, p_all{INFINITY, INT_MAX};
-  for (int k = 0; k < p.NCS; ++k) {
-    const RacePartial* src = p.race_part + (size_t)i * p.NCS + k;
-    KeyState kr{__ldcg(&src->key_r), __ldcg(&src->idx_r)};
-    KeyState kp{__ldcg(&src->key_p), __ldcg(&src->idx_p)};
-    if (key_better(kr, r_all)) r_all = kr;
-    if (key_better(kp, p_all)) p_all = kp;
+  if (threadIdx.x == 0) {
+    KeyState r_all{INFINITY, INT_MAX}, p_all{INFINITY, INT_MAX};
+    for (int k = 0; k < p.NCS; ++k) {
+      const RacePartial* src = p.race_part + (size_t)i * p.NCS + k;
+      KeyState kr{__ldcg(&src->key_r), __ldcg(&src->idx_r)};
+      KeyState kp{__ldcg(&src->key_p), __ldcg(&src->idx_p)};
+      if (key_better(kr, r_all)) r_all = kr;
+      if (key_better(kp, p_all)) p_all = kp;
+    }
+    p.counters[i] = 0u;  // leave the workspace zeroed for the next call
+    // bonus: race on p_n; one-hot rejection with an empty residual: race on p
+    sh_y = r_all.idx != INT_MAX ? r_all.idx : (general_q ? -2 : p_all.idx);
   }
-  p.counters[i] = 0u;  // leave the workspace zeroed for the next call
-  if (bad) return;
-  int y = r_all.idx;
-  if (!rejected) y = r_all.idx;                 // bonus: race on p_n
-  else if (y == INT_MAX) y = p_all.idx;         // empty residual: draw from p
+  __syncthreads();
+  int y = sh_y;
+  if (y == -2) {
+    // Residual max(0, p - q) empty in fp32 (p <= q everywhere): draw from p.
+    // The whole row in this CTA; this happens only when p and q agree to
+    // rounding at a rejection.
+    KeyState bp{INFINITY, INT_MAX}, unused{INFINITY, INT_MAX};
+    if (p.vec_s)
+      race_chunk_vec<T, T, false>(row, nullptr, -1, 0, V, c2, rec.M2, rec.invS, rec.position, req, k0, k1, bp,
+                                  unused);
+    else
+      race_chunk_scalar<T, false>(row, nullptr, p.q_dtype, -1, 0, V, c2, rec.M2, rec.invS, rec.position, req, k0,
+                                  k1, bp, unused);
+    bp = cta_min_key(bp, sh_red);
+    y = bp.idx;
+  }
+  if (threadIdx.x != 0) return;
+  int32_t* tok = p.out_tokens + (size_t)i * (p.K + 1);
   if (y == INT_MAX) {
     report(p.status, SPEC_ERR_BAD_INPUT);
-    tok[a] = -1;
+    tok[rec.a] = -1;
     p.accepted_len[i] = 0;
     return;
   }
-  tok[a] = y;
+  tok[rec.a] = y;
 }
 
 // ---------------------------------------------------------------------------
@@ -619,10 +816,7 @@ template <typename T>
 static cudaError_t launch_typed(const VerifyLaunch& p, cudaStream_t stream, cudaEvent_t ev_before,
                                 cudaEvent_t ev_after) {
   const bool greedy = p.temperature == 0.0f;
-  VerifyLaunch pd = p;
-  if (greedy) pd.NCS = 1;  // no sampling pass: one decision CTA per request
-  const unsigned grid1 = (unsigned)((long long)p.R_max * p.NC);
-  const unsigned grid2 = (unsigned)((long long)p.B * pd.NCS);
+  const unsigned grid1 = (unsigned)((long long)p.B * (p.K + 1) * p.NC);
   if (ev_before) cudaEventRecord(ev_before, stream);
   if (greedy)
     stream_rows_kernel<T, true><<<grid1, kStreamThreads, 0, stream>>>(p);
@@ -631,10 +825,9 @@ static cudaError_t launch_typed(const VerifyLaunch& p, cudaStream_t stream, cuda
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   if (ev_after) cudaEventRecord(ev_after, stream);
-  if (greedy)
-    decide_sample_kernel<T, true><<<grid2, kSampleThreads, 0, stream>>>(pd);
-  else
-    decide_sample_kernel<T, false><<<grid2, kSampleThreads, 0, stream>>>(pd);
+  if (greedy) return cudaSuccess;
+  const unsigned grid2 = (unsigned)((long long)p.B * p.NCS);
+  sample_kernel<T><<<grid2, kSampleThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 
