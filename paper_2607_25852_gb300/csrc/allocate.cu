@@ -16,6 +16,7 @@
 // exactly; the first maximiser of U / cost is chosen and the kept prefixes
 // are packed densely.
 #include <float.h>
+#include <limits.h>
 #include <math.h>
 
 #include <algorithm>
@@ -56,9 +57,10 @@ __device__ __forceinline__ long long block_inclusive_scan(long long x, long long
   return x + before;
 }
 
-// Shared-memory layout (dynamic): two key buffers of N entries, then the
-// confidences [B*K] fp32, then the draft tokens [B*K] int32, then
-// last_tokens [B] int32 and pos_base [B] int64.
+// Shared-memory layout (dynamic): two key buffers of N entries, then
+// pos_base [B] int64, the confidences [B][K] fp32 at the odd row stride K | 1
+// (so that the threads of a warp, one request each, read distinct banks), the
+// draft tokens [B*K] int32 and last_tokens [B] int32.
 struct AllocSmem {
   unsigned long long* keys[2];
   float* conf;
@@ -75,7 +77,7 @@ __device__ __forceinline__ AllocSmem carve(unsigned char* base, int N, int BK, i
   s.pos = reinterpret_cast<long long*>(p);
   p += (size_t)B * 8;
   s.conf = reinterpret_cast<float*>(p);
-  p += (size_t)BK * 4;
+  p += BK > 0 ? (size_t)(BK + B) * 4 : 0;
   s.drafts = reinterpret_cast<int32_t*>(p);
   p += (size_t)BK * 4;
   s.last = reinterpret_cast<int32_t*>(p);
@@ -84,12 +86,15 @@ __device__ __forceinline__ AllocSmem carve(unsigned char* base, int N, int BK, i
 
 size_t allocate_smem_bytes(int B, int K) {
   const size_t N = (size_t)B * (K + 1), BK = (size_t)B * K;
-  return N * 16 + (size_t)B * 8 + BK * 8 + (size_t)B * 4 + 16;
+  // at most 24 N + 8 B + 16 bytes <= 229,392 for N <= 8192 (K = 0 needs no
+  // confidences: 16 N + 12 B + 16)
+  return N * 16 + (size_t)B * 8 + (BK > 0 ? (BK + B) * 4 : 0) + BK * 4 + (size_t)B * 4 + 16;
 }
 
 __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaunch p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int B = p.B, K = p.K, N = B * (K + 1), BK = B * K, L0 = K + 1;
+  const int CS = K | 1;  // odd row stride of the staged confidences
   const AllocSmem sm = carve(smem_raw, N, BK, B);
   __shared__ long long warp_tot[32];
   __shared__ int sh_best_c;
@@ -99,7 +104,8 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
 
   // ---- every global input in one round trip, coalesced ----
   for (int q = tid; q < BK; q += kAllocThreads) {
-    sm.conf[q] = p.conf[q];
+    const int i = q / K;
+    sm.conf[q + i * (CS - K)] = p.conf[q];  // [i][k] at i * CS + k
     sm.drafts[q] = p.drafts[q];
   }
   for (int i = tid; i < B; i += kAllocThreads) {
@@ -113,7 +119,7 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
     float s = 1.0f;
     sm.keys[0][i * L0] = position_key(s, 0, i);
     for (int k = 1; k <= K; ++k) {
-      float c = sm.conf[i * K + (k - 1)];
+      float c = sm.conf[i * CS + (k - 1)];
       if (!(c >= 0.0f && c <= 1.0f)) {
         sh_bad = 1;
         c = 0.0f;
@@ -125,30 +131,30 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
   __syncthreads();
 
   // ---- merge tree over the B sorted runs (descending) ----
+  // Level l merges runs of L = L0 * 2^l keys; position e lies in run
+  // (e / L0) >> l.  N <= 8192, so 32-bit indices suffice.
   int cur = 0;
-  for (long long L = L0; L < N; L *= 2) {
+  for (int lev = 0, L = L0; L < N; ++lev, L *= 2) {
     const unsigned long long* in = sm.keys[cur];
     unsigned long long* out = sm.keys[cur ^ 1];
     for (int e = tid; e < N; e += kAllocThreads) {
-      const long long run = e / L;
-      const long long start = run * L;
-      const long long partner = run ^ 1;
-      const long long pstart = partner * L;
+      const int run = (e / L0) >> lev;
+      const int start = run * L;
+      const int pstart = (run ^ 1) * L;
       const unsigned long long x = in[e];
       if (pstart >= N) {  // unpaired last run: copied through
         out[e] = x;
         continue;
       }
-      const long long plen = min((long long)N, pstart + L) - pstart;
+      const int plen = min(N, pstart + L) - pstart;
       // number of partner keys greater than x (the partner run is descending)
-      int lo = 0, hi = (int)plen;
+      int lo = 0, hi = plen;
       while (lo < hi) {
         const int mid = (lo + hi) >> 1;
         if (in[pstart + mid] > x) lo = mid + 1;
         else hi = mid;
       }
-      const long long base = min(start, pstart);
-      out[base + (e - start) + lo] = x;
+      out[min(start, pstart) + (e - start) + lo] = x;
     }
     __syncthreads();
     cur ^= 1;
@@ -172,21 +178,29 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
 
   // ---- Eq. (dcut-select): first maximiser of U / cost ----
   if (tid < 32) {
-    // utilities in parallel, argmax by lane 0 in candidate order
-    for (int c = tid; c < p.M; c += 32)
-      if (p.utility_out) p.utility_out[c] = ldexp((double)prefix[p.cand_T[c] - 1], -40);
-    if (tid == 0) {
-      int best_c = 0;
-      double best_obj = -INFINITY;
-      for (int c = 0; c < p.M; ++c) {
-        const double obj = ldexp((double)prefix[p.cand_T[c] - 1], -40) / p.cand_cost[c];
-        if (obj > best_obj) {
-          best_obj = obj;
-          best_c = c;
-        }
+    // one lane per candidate (M <= 64: two per lane); the first maximiser
+    // in candidate order wins ties, as a sequential scan would
+    double best_obj = -INFINITY;
+    int best_c = INT_MAX;
+    for (int c = tid; c < p.M; c += 32) {
+      const double U = ldexp((double)prefix[p.cand_T[c] - 1], -40);
+      if (p.utility_out) p.utility_out[c] = U;
+      const double obj = U / p.cand_cost[c];
+      if (obj > best_obj) {  // c increases along the lane's loop
+        best_obj = obj;
+        best_c = c;
       }
-      sh_best_c = best_c;
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const double ob = __shfl_xor_sync(0xFFFFFFFFu, best_obj, o);
+      const int cb = __shfl_xor_sync(0xFFFFFFFFu, best_c, o);
+      if (ob > best_obj || (ob == best_obj && cb < best_c)) {
+        best_obj = ob;
+        best_c = cb;
+      }
+    }
+    if (tid == 0) sh_best_c = best_c == INT_MAX ? 0 : best_c;
   }
   __syncthreads();
   const int T = p.cand_T[sh_best_c];

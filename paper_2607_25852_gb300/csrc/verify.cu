@@ -39,6 +39,7 @@ constexpr int kStreamThreads = 256;
 constexpr int kUnroll = 4;
 constexpr int kSampleThreads = 256;
 constexpr int kMaxRows = SPEC_MAX_DRAFTS + 1;
+constexpr unsigned long long kCopyWaitNs = 2000000000ull;  // bound on one bulk-copy wait (2 s)
 
 static inline long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
 static inline long long round_up(long long a, long long b) { return ceil_div(a, b) * b; }
@@ -379,6 +380,9 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
   const int c = rem - j * p.NC;
   const ReqShape rs = request_shape(p, i);
   if (!(rs.valid ? j <= rs.n : (j == 0 && c == 0))) return;
+  // The sampling kernel may start launching once every CTA here has started;
+  // it waits for this grid's completion before it reads anything.
+  pdl_launch_dependents();
   __shared__ int sh_last;
   if (rs.valid) {
     const long long r = rs.row0 + j;
@@ -555,13 +559,27 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
 // ---------------------------------------------------------------------------
 // Sampling pass (t > 0)
 // ---------------------------------------------------------------------------
-// Eight consecutive entries of a row as floats, from 16-byte loads.
+// Eight consecutive entries of a row as floats, from 16-byte loads: from
+// global memory (streaming) or from a chunk staged in shared memory.
+template <bool kShared>
+__device__ __forceinline__ uint4 load16(const void* ptr) {
+  if (kShared) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"((uint32_t)__cvta_generic_to_shared(ptr)));
+    return v;
+  }
+  return ldg_stream(ptr);
+}
+
 template <typename T>
 struct Row8;
 template <>
 struct Row8<__nv_bfloat16> {
+  template <bool kShared>
   __device__ static void load(const void* row, int g8, float x[8]) {
-    const uint4 w = ldg_stream(static_cast<const uint4*>(row) + g8);
+    const uint4 w = load16<kShared>(static_cast<const uint4*>(row) + g8);
     x[0] = bf16_lo(w.x);
     x[1] = bf16_hi(w.x);
     x[2] = bf16_lo(w.y);
@@ -574,9 +592,10 @@ struct Row8<__nv_bfloat16> {
 };
 template <>
 struct Row8<float> {
+  template <bool kShared>
   __device__ static void load(const void* row, int g8, float x[8]) {
-    const uint4 a = ldg_stream(static_cast<const uint4*>(row) + 2 * g8);
-    const uint4 b = ldg_stream(static_cast<const uint4*>(row) + 2 * g8 + 1);
+    const uint4 a = load16<kShared>(static_cast<const uint4*>(row) + 2 * g8);
+    const uint4 b = load16<kShared>(static_cast<const uint4*>(row) + 2 * g8 + 1);
     x[0] = __uint_as_float(a.x);
     x[1] = __uint_as_float(a.y);
     x[2] = __uint_as_float(a.z);
@@ -624,8 +643,10 @@ __device__ __forceinline__ float warp_thr24(const KeyState& best) {
 // does not change the argmin), the excluded draft token z_excl into best_p and
 // every other entry into best_r.
 // Vector form: 16-byte loads, groups of 8 entries (two Philox blocks) per
-// thread and step; needs v0, v1 multiples of 8 and aligned rows.
-template <typename T, typename Q, bool kGeneral>
+// thread and step; needs v0, v1 multiples of 8 and aligned rows.  kShared:
+// row and qrow point at entry v0 of chunks staged in shared memory; otherwise
+// at entry 0 of the rows in global memory.
+template <typename T, typename Q, bool kGeneral, bool kShared = false>
 __device__ __forceinline__ void race_chunk_vec(const void* row, const void* qrow, int z_excl, int v0, int v1,
                                                float c2, float M2, float invS, uint32_t position,
                                                uint64_t req, uint32_t k0, uint32_t k1, KeyState& best_r,
@@ -633,8 +654,9 @@ __device__ __forceinline__ void race_chunk_vec(const void* row, const void* qrow
   float thr24 = best_r.key * 0x1p24f;
   for (int g8 = (v0 >> 3) + threadIdx.x; g8 * 8 < v1; g8 += kSampleThreads) {
     float x[8], qv[8];
-    Row8<T>::load(row, g8, x);
-    if (kGeneral) Row8<Q>::load(qrow, g8, qv);
+    const int gi = kShared ? g8 - (v0 >> 3) : g8;
+    Row8<T>::template load<kShared>(row, gi, x);
+    if (kGeneral) Row8<Q>::template load<kShared>(qrow, gi, qv);
     const uint4 r0 = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)(2 * g8)), k0, k1);
     const uint4 r1 = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)(2 * g8 + 1)), k0, k1);
     const uint32_t words[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
@@ -703,11 +725,23 @@ __device__ __forceinline__ KeyState cta_min_key(KeyState b, KeyState* sh) {
   return b;
 }
 
+// Dynamic shared memory of the sampling kernel: the logits chunk, then the q
+// chunk, each at a 128-byte boundary (16-byte loads path only).
+size_t sample_stage_bytes(const VerifyLaunch& p) {
+  if (!p.vec_s) return 0;
+  const size_t esize = p.logits_dtype == SPEC_F32 ? 4 : 2, qsize = p.q_dtype == SPEC_F32 ? 4 : 2;
+  const size_t lb = ((size_t)p.chunk_s * esize + 127) / 128 * 128;
+  return lb + (p.q ? (size_t)p.chunk_s * qsize : 0);
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyLaunch p) {
+  extern __shared__ __align__(128) unsigned char stage[];
+  __shared__ uint64_t sh_bar;
   const int i = blockIdx.x / p.NCS;
   const int cs = blockIdx.x - i * p.NCS;
   const int V = p.V;
+  pdl_wait_prerequisites();  // the decisions of the streaming kernel
   const ReqRec rec = p.req_rec[i];
   if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
   const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
@@ -729,7 +763,38 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   {
     const int v0 = cs * p.chunk_s;
     const int v1 = min(V, v0 + p.chunk_s);
-    if (p.vec_s) {
+    if (p.stage_s) {
+      // Stage the chunk (and the q chunk) in shared memory with bulk copies:
+      // one round trip per CTA instead of one per group of 8 entries.
+      const uint32_t lbytes = (uint32_t)(v1 - v0) * (uint32_t)sizeof(T);
+      const uint32_t qbytes = general_q ? (uint32_t)(v1 - v0) * (uint32_t)qsize : 0u;
+      unsigned char* lstage = stage;
+      unsigned char* qstage = stage + ((size_t)p.chunk_s * sizeof(T) + 127) / 128 * 128;
+      if (threadIdx.x == 0) {
+        mbar_init(&sh_bar, 1);
+        mbar_init_fence();
+        mbar_arrive_tx(&sh_bar, lbytes + qbytes);
+        bulk_load(lstage, row + v0, lbytes, &sh_bar);
+        if (general_q) bulk_load(qstage, (const char*)qrow + (size_t)v0 * qsize, qbytes, &sh_bar);
+      }
+      __syncthreads();  // the barrier is initialised before anyone waits on it
+      if (!mbar_wait_bounded(&sh_bar, 0, kCopyWaitNs)) {
+        // The copy did not land: report it, give it a second bounded wait so
+        // that it does not write into a finished CTA, and skip the race.
+        if (threadIdx.x == 0) report(p.status, SPEC_ERR_TIMEOUT);
+        mbar_wait_bounded(&sh_bar, 0, kCopyWaitNs);
+      } else if (general_q) {
+        if (p.q_dtype == SPEC_F32)
+          race_chunk_vec<T, float, true, true>(lstage, qstage, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
+                                               rec.position, req, k0, k1, best_r, best_p);
+        else
+          race_chunk_vec<T, __nv_bfloat16, true, true>(lstage, qstage, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
+                                                       rec.position, req, k0, k1, best_r, best_p);
+      } else {
+        race_chunk_vec<T, T, false, true>(lstage, nullptr, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position,
+                                          req, k0, k1, best_r, best_p);
+      }
+    } else if (p.vec_s) {
       if (general_q) {
         if (p.q_dtype == SPEC_F32)
           race_chunk_vec<T, float, true>(row, qrow, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position, req,
@@ -826,8 +891,25 @@ static cudaError_t launch_typed(const VerifyLaunch& p, cudaStream_t stream, cuda
   if (err != cudaSuccess) return err;
   if (ev_after) cudaEventRecord(ev_after, stream);
   if (greedy) return cudaSuccess;
-  const unsigned grid2 = (unsigned)((long long)p.B * p.NCS);
-  sample_kernel<T><<<grid2, kSampleThreads, 0, stream>>>(p);
+  const size_t smem = p.stage_s ? sample_stage_bytes(p) : 0;
+  if (smem > 48 * 1024) {
+    err = cudaFuncSetAttribute(sample_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (err != cudaSuccess) return err;
+  }
+  // Programmatic dependent launch: the sampling CTAs are launched while the
+  // streaming kernel drains and wait (griddepcontrol.wait) for its completion.
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)((long long)p.B * p.NCS));
+  cfg.blockDim = dim3(kSampleThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = cudaLaunchKernelEx(&cfg, sample_kernel<T>, p);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
