@@ -38,8 +38,10 @@
  * with key = (lo32(seed_i), hi32(seed_i)) and counter =
  *   (lo32(position), lo32(request_id_i), hi32(request_id_i), purpose<<28 | sub)
  *   SPEC_PURPOSE_ACCEPT: sub = 0; u = (word0 >> 8) * 2^-24 in [0, 1)
- *   SPEC_PURPOSE_SAMPLE: sub = v >> 2; E_v = -ln((2 * (word[v & 3] >> 9) + 1) * 2^-24),
- *                        the midpoint of one of 2^23 cells of (0, 1), so E_v > 0
+ *   SPEC_PURPOSE_SAMPLE:          sub = b >> 2; block variate E_b from word[b & 3]
+ *   SPEC_PURPOSE_SAMPLE_IN_BLOCK: sub = v >> 2; entry variate E'_v from word[v & 3]
+ * where a word x gives E = -ln((2 * (x >> 9) + 1) * 2^-24), the midpoint of
+ * one of 2^23 cells of (0, 1), so E > 0;
  * so a round replays bit for bit from (seed, request id, position).
  */
 #ifndef SPEC_H_
@@ -71,6 +73,7 @@ typedef enum { SPEC_BF16 = 0, SPEC_F32 = 1 } spec_dtype;
 
 #define SPEC_PURPOSE_ACCEPT 1u
 #define SPEC_PURPOSE_SAMPLE 2u
+#define SPEC_PURPOSE_SAMPLE_IN_BLOCK 3u
 
 /* Limits checked on the host (SPEC_ERR_INVALID_ARG beyond them). */
 #define SPEC_MAX_VOCAB (1 << 30)       /* V < 2^30 keeps v >> 2 within 28 bits */
@@ -150,10 +153,13 @@ int spec_allocate(const float* conf, int B, int K, const int32_t* cand_T,
  *           u_j < min(1, p_j(z_{j+1}) / q_j(z_{j+1}))   (q_j(z) = 0 gives 1
  *           if p_j(z) > 0); at the first rejection a = j and y is drawn from
  *           max(0, p_a - q_a) (from p_a if that is identically zero); if all
- *           n are accepted, a = n and y is drawn from p_n.  The draw is the
- *           exponential race y = argmin_{w_v > 0} E_v / w_v (lowest v on
- *           ties), an exact sampler of w / sum(w) that does not depend on
- *           summation order.
+ *           n are accepted, a = n and y is drawn from p_n.  The draw is a
+ *           two-level exponential race: with blocks of 256 consecutive
+ *           entries and W_b = sum_{v in b} w_v, first
+ *           b* = argmin_{W_b > 0} E_b / W_b, then
+ *           y = argmin_{v in b*, w_v > 0} E'_v / w_v (lowest index on ties
+ *           at both levels): an exact sampler of w / sum(w), since
+ *           P(b*) = W_b / W and P(y | b*) = w_y / W_b.
  *   out_tokens[i] = z_1..z_a, y, then -1 up to K+1 entries.
  * Arguments
  *   logits          device [R, V] of logits_dtype, rows of request i at

@@ -46,7 +46,7 @@ def _declare(lib):
     lib.oracle_philox4x32_10.restype = None
     lib.oracle_accept_uniform.argtypes = [ctypes.c_uint64] * 3
     lib.oracle_accept_uniform.restype = ctypes.c_double
-    lib.oracle_race_exponential.argtypes = [ctypes.c_uint64] * 3 + [ctypes.c_uint32]
+    lib.oracle_race_exponential.argtypes = [ctypes.c_uint64] * 3 + [ctypes.c_uint32, ctypes.c_int]
     lib.oracle_race_variate.argtypes = [ctypes.c_uint32]
     lib.oracle_race_variate.restype = ctypes.c_double
     lib.oracle_race_exponential.restype = ctypes.c_double
@@ -116,8 +116,13 @@ def race_variate(word: int) -> float:
     return load().oracle_race_variate(word)
 
 
-def race_exponential(seed: int, request: int, position: int, v: int) -> float:
-    return load().oracle_race_exponential(seed, request, position, v)
+def race_exponential(seed: int, request: int, position: int, index: int, level: int = 2) -> float:
+    """Race variate of block `index` (level 1) or entry `index` (level 2)."""
+    return load().oracle_race_exponential(seed, request, position, index, level)
+
+
+# Layout of the race record (9 values per request).
+RACE_FIELDS = ("block_key", "block", "block2_key", "block2", "y", "y_key", "y2_key", "y2", "y_in_block2")
 
 
 def row_stats(row, t: float):
@@ -144,7 +149,7 @@ def verify_request(logits, drafts, q, t, seed, request, pos_base):
         accepted=np.zeros(1, np.int32), tokens=np.zeros(n + 1, np.int32),
         p_draft=np.zeros(max(n, 1), np.float64), row_m=np.zeros(n + 1, np.float64),
         row_logS=np.zeros(n + 1, np.float64), u=np.zeros(max(n, 1), np.float64),
-        r=np.zeros(max(n, 1), np.float64), race=np.zeros(4, np.float64),
+        r=np.zeros(max(n, 1), np.float64), race=np.zeros(9, np.float64),
         mode=np.zeros(1, np.int32))
     st = load().oracle_verify_request(
         _ptr(logits), _dtype_code(logits), _ptr(drafts), _ptr(q), _dtype_code(q),
@@ -185,7 +190,7 @@ def verify_batch(logits, drafts, q, t, seeds, request_ids, pos_base,
         accepted=np.zeros(B, np.int32), tokens=np.full((B, K + 1), -1, np.int32),
         p_draft=np.zeros((B, K), np.float64), row_m=np.zeros(R, np.float64),
         row_logS=np.zeros(R, np.float64), u=np.zeros((B, K), np.float64),
-        r=np.zeros((B, K), np.float64), race=np.zeros((B, 4), np.float64),
+        r=np.zeros((B, K), np.float64), race=np.zeros((B, 9), np.float64),
         mode=np.zeros(B, np.int32), status=np.zeros(B, np.int32))
     lib = load()
     if requests is None:

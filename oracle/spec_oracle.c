@@ -27,8 +27,13 @@
  *   - row j of a request verifies draft z_{j+1}; the bonus row is row n;
  *   - accept iff u < r with u in [0,1);
  *   - uniforms come from Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11)
- *     with the counter layout below; the draw from a weight vector w is the
- *     exponential race y = argmin_{v: w_v > 0} E_v / w_v (ties to lowest v);
+ *     with the counter layout below; the draw from a weight vector w is a
+ *     two-level exponential race: entries are grouped in blocks of 256
+ *     consecutive indices with block weights W_b = sum_{v in b} w_v; the block
+ *     b* = argmin_{W_b > 0} E_b / W_b is drawn first, then the entry
+ *     y = argmin_{v in b*, w_v > 0} E'_v / w_v (ties to the lowest index at
+ *     both levels).  Each level is an exact draw (P(b*) = W_b / W,
+ *     P(y | b*) = w_y / W_b), so P(y) = w_y / W;
  *   - temperature 0 is the longest argmax-matching prefix plus the argmax of
  *     the first unmatched row (ties to lowest index);
  *   - allocator scores are fp32 products taken in order k = 1..K (the
@@ -38,8 +43,9 @@
  *
  * Counter layout (frozen): key = (lo32(seed), hi32(seed));
  *   counter = (lo32(position), lo32(request), hi32(request), purpose<<28 | sub)
- *   purpose ACCEPT = 1 (sub = 0, word 0 used), SAMPLE = 2 (sub = v / 4,
- *   word v % 4 used).  Acceptance uniform: (x >> 8) * 2^-24.  Race variate:
+ *   purpose ACCEPT = 1 (sub = 0, word 0 used), SAMPLE = 2 (block variates:
+ *   sub = b / 4, word b % 4), SAMPLE_IN_BLOCK = 3 (entry variates: sub = v / 4,
+ *   word v % 4).  Acceptance uniform: (x >> 8) * 2^-24.  Race variate:
  *   E = -ln((2 * (x >> 9) + 1) * 2^-24), the midpoint of one of 2^23 equal
  *   cells of (0, 1), so that E > 0: a variate of exactly 0 would make its entry
  *   win whatever its weight, and the draw would no longer follow w / sum(w).
@@ -66,6 +72,8 @@
 
 #define OR_PURPOSE_ACCEPT 1u
 #define OR_PURPOSE_SAMPLE 2u
+#define OR_PURPOSE_SAMPLE_IN_BLOCK 3u
+#define OR_RACE_BLOCK 256
 
 /* ------------------------------------------------------------------------ */
 /* Element access.  bf16 is the upper half of an IEEE binary32 word.        */
@@ -139,12 +147,77 @@ double oracle_race_variate(uint32_t word) {
   return -log(u);
 }
 
-/* Exponential variate E_v of the sampling race at `position`, entry v. */
+/* Exponential variate of the sampling race at `position`: level 1 (block b,
+ * level = 1) or level 2 (entry v, level = 2). */
 double oracle_race_exponential(uint64_t seed, uint64_t request,
-                               uint64_t position, uint32_t v) {
+                               uint64_t position, uint32_t index, int level) {
   uint32_t w[4];
-  draw_words(seed, request, position, OR_PURPOSE_SAMPLE, v >> 2, w);
-  return oracle_race_variate(w[v & 3u]);
+  draw_words(seed, request, position,
+             level == 1 ? OR_PURPOSE_SAMPLE : OR_PURPOSE_SAMPLE_IN_BLOCK,
+             index >> 2, w);
+  return oracle_race_variate(w[index & 3u]);
+}
+
+/* Two-level exponential race over weights w[0..V) (see the file header).
+ * race_out[9]: best block key, best block, second block key, second block,
+ * the winner y in the best block, its key, the second key in that block, the
+ * second entry in that block, and the winner in the second block (-1 if
+ * none).  Returns y, or -1 if every weight is zero. */
+static int two_level_race(const double* w, int V, uint64_t seed,
+                          uint64_t request, uint64_t position,
+                          double* race_out) {
+  const int nb = (V + OR_RACE_BLOCK - 1) / OR_RACE_BLOCK;
+  double b1k = INFINITY, b2k = INFINITY;
+  int b1 = -1, b2 = -1;
+  for (int b = 0; b < nb; ++b) {
+    double W = 0.0;
+    for (int v = b * OR_RACE_BLOCK; v < V && v < (b + 1) * OR_RACE_BLOCK; ++v)
+      W += w[v];
+    if (!(W > 0.0)) continue;
+    double key = oracle_race_exponential(seed, request, position, (uint32_t)b, 1) / W;
+    if (key < b1k) {
+      b2k = b1k;
+      b2 = b1;
+      b1k = key;
+      b1 = b;
+    } else if (key < b2k) {
+      b2k = key;
+      b2 = b;
+    }
+  }
+  double yk[2] = {INFINITY, INFINITY}, y2k = INFINITY;
+  int y[2] = {-1, -1}, y2 = -1;
+  for (int pass = 0; pass < 2; ++pass) {
+    int b = pass == 0 ? b1 : b2;
+    if (b < 0) continue;
+    for (int v = b * OR_RACE_BLOCK; v < V && v < (b + 1) * OR_RACE_BLOCK; ++v) {
+      if (!(w[v] > 0.0)) continue;
+      double key = oracle_race_exponential(seed, request, position, (uint32_t)v, 2) / w[v];
+      if (key < yk[pass]) {
+        if (pass == 0) {
+          y2k = yk[0];
+          y2 = y[0];
+        }
+        yk[pass] = key;
+        y[pass] = v;
+      } else if (pass == 0 && key < y2k) {
+        y2k = key;
+        y2 = v;
+      }
+    }
+  }
+  if (race_out) {
+    race_out[0] = b1k;
+    race_out[1] = b1;
+    race_out[2] = b2k;
+    race_out[3] = b2;
+    race_out[4] = y[0];
+    race_out[5] = yk[0];
+    race_out[6] = y2k;
+    race_out[7] = y2;
+    race_out[8] = y[1];
+  }
+  return y[0];
 }
 
 /* ------------------------------------------------------------------------ */
@@ -211,7 +284,7 @@ void oracle_row_stats(const void* row, int dtype, int V, double t,
 /*   p_draft_out[n] : p_j(z_{j+1})                                          */
 /*   row_m_out, row_logS_out [n+1] : m_j and ln S_j (t > 0); max l and 0    */
 /*   u_out, r_out [n] : acceptance uniform and ratio per draft (t > 0)      */
-/*   race_out[4]    : best key, index of best, second key, index of second  */
+/*   race_out[9]    : the two-level race record (two_level_race)             */
 /*   mode_out       : OR_MODE_*                                             */
 /* Returns OR_OK, or OR_ERR_BAD_INPUT (then a = 0 and tokens[0] = -1).      */
 /* ------------------------------------------------------------------------ */
@@ -226,10 +299,7 @@ int oracle_verify_request(const void* logits, int logits_dtype,
   for (int j = 0; j <= n; ++j) tokens_out[j] = -1;
   *accepted_out = 0;
   if (race_out) {
-    race_out[0] = INFINITY;
-    race_out[1] = -1;
-    race_out[2] = INFINITY;
-    race_out[3] = -1;
+    for (int k = 0; k < 9; ++k) race_out[k] = (k == 0 || k == 2 || k == 5 || k == 6) ? INFINITY : -1;
   }
   if (mode_out) *mode_out = t == 0.0 ? OR_MODE_GREEDY : OR_MODE_BONUS;
 
@@ -335,23 +405,9 @@ int oracle_verify_request(const void* logits, int logits_dtype,
       w[v] = row_prob(ROW(row), logits_dtype, v, t, m[row], S[row]);
   }
 
-  /* Exponential race: y = argmin_{w_v > 0} E_v / w_v, lowest v on ties. */
-  double best = INFINITY, second = INFINITY;
-  int best_v = -1, second_v = -1;
+  /* Two-level exponential race over w at the sampled position. */
   const uint64_t position = (uint64_t)(pos_base + row);
-  for (int v = 0; v < V; ++v) {
-    if (!(w[v] > 0.0)) continue;
-    double key = oracle_race_exponential(seed, request, position, (uint32_t)v) / w[v];
-    if (key < best) {
-      second = best;
-      second_v = best_v;
-      best = key;
-      best_v = v;
-    } else if (key < second) {
-      second = key;
-      second_v = v;
-    }
-  }
+  int best_v = two_level_race(w, V, seed, request, position, race_out);
   if (best_v < 0) {
     status = OR_ERR_BAD_INPUT;
     goto done;
@@ -360,12 +416,6 @@ int oracle_verify_request(const void* logits, int logits_dtype,
   tokens_out[a] = best_v;
   *accepted_out = a;
   if (mode_out) *mode_out = mode;
-  if (race_out) {
-    race_out[0] = best;
-    race_out[1] = best_v;
-    race_out[2] = second;
-    race_out[3] = second_v;
-  }
 
 done:
   if (status != OR_OK) {
@@ -424,7 +474,7 @@ int oracle_verify_batch(const void* logits, int logits_dtype,
           row_logS_out ? row_logS_out + row0 : NULL,
           u_out ? u_out + (size_t)i * K : NULL,
           r_out ? r_out + (size_t)i * K : NULL,
-          race_out ? race_out + (size_t)i * 4 : NULL,
+          race_out ? race_out + (size_t)i * 9 : NULL,
           mode_out ? mode_out + i : NULL);
     }
     if (status_out) status_out[i] = st;

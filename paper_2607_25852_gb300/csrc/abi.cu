@@ -175,7 +175,6 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
     const size_t esize = logits_dtype == SPEC_F32 ? 4 : 2, qsize = q_dtype == SPEC_F32 ? 4 : 2;
     const bool q_ok = p.q == nullptr || (reinterpret_cast<uintptr_t>(p.q) % 16 == 0 && (V * qsize) % 16 == 0);
     p.vec_s = V % 8 == 0 && reinterpret_cast<uintptr_t>(logits) % 16 == 0 && (V * esize) % 16 == 0 && q_ok;
-    p.stage_s = p.vec_s && spec::sample_stage_bytes(p) <= spec::kMaxSampleStageBytes;
   }
   return spec::launch_verify(p, stream, ev_before, ev_after) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }

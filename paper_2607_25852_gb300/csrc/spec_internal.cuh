@@ -219,7 +219,6 @@ struct VerifyLaunch {
   int NCS;                // vocabulary chunks per request, sampling pass
   int chunk_s;            // elements per sampling chunk (multiple of 8)
   bool vec_s;             // sampling pass may use 16-byte loads
-  bool stage_s;           // sampling pass stages its chunks in shared memory (implies vec_s)
 };
 
 struct AllocLaunch {
@@ -261,9 +260,6 @@ struct VerifyGeometry {
 VerifyGeometry verify_geometry(int B, int K, int V);
 
 // Launchers (return cudaSuccess or the launch error).
-// Shared memory the sampling kernel needs to stage one chunk (and its q chunk).
-size_t sample_stage_bytes(const VerifyLaunch& p);
-constexpr size_t kMaxSampleStageBytes = 110 * 1024;  // two sampling CTAs per SM at most this large
 cudaError_t launch_verify(const VerifyLaunch& p, cudaStream_t stream, cudaEvent_t ev_before,
                           cudaEvent_t ev_after);
 cudaError_t launch_allocate(const AllocLaunch& p, cudaStream_t stream);

@@ -39,7 +39,6 @@ constexpr int kStreamThreads = 256;
 constexpr int kUnroll = 4;
 constexpr int kSampleThreads = 256;
 constexpr int kMaxRows = SPEC_MAX_DRAFTS + 1;
-constexpr unsigned long long kCopyWaitNs = 2000000000ull;  // bound on one bulk-copy wait (2 s)
 
 static inline long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
 static inline long long round_up(long long a, long long b) { return ceil_div(a, b) * b; }
@@ -52,10 +51,12 @@ VerifyGeometry verify_geometry(int B, int K, int V) {
   nc = std::max(1LL, std::min(nc, std::max(1LL, (long long)V / 4096)));
   long long chunk = round_up(ceil_div(V, nc), 8);
   nc = ceil_div(V, chunk);  // every chunk non-empty
-  // Sampling pass: aim for ~1024 (request, chunk) items of >= 2048 elements.
-  long long ncs = ceil_div(1024, B);
+  // Sampling pass: aim for ~560 (request, chunk) CTAs, about one resident
+  // wave on 152 SMs, of >= 2048 elements each, every chunk a whole number of
+  // race quads (1024 entries).
+  long long ncs = ceil_div(560, B);
   ncs = std::max(1LL, std::min(ncs, std::max(1LL, (long long)V / 2048)));
-  long long chunk_s = round_up(ceil_div(V, ncs), 8);
+  long long chunk_s = round_up(ceil_div(V, ncs), 1024);
   ncs = ceil_div(V, chunk_s);
   g.NC = (int)nc;
   g.chunk = (int)chunk;
@@ -607,104 +608,155 @@ struct Row8<float> {
   }
 };
 
-// Exponential race entries.  The race variate of a Philox word is
-// E = -ln(u), u = (2 * (word >> 9) + 1) * 2^-24; with m = 2^24 * (1 - u), an
-// odd integer below 2^24, E = -ln(1 - m * 2^-24) exactly as in the oracle.
+// ---------------------------------------------------------------------------
+// Two-level exponential race
+// ---------------------------------------------------------------------------
+// The draw from weights w is made in two exact steps: the level-1 block
+// b* = argmin_{W_b > 0} E_b / W_b over blocks of kRaceBlock consecutive
+// entries (W_b = sum_{v in b} w_v), then y = argmin_{v in b*, w_v > 0} E'_v / w_v
+// (ties to the lowest index).  Level 1 needs one variate per block, so the
+// Philox work is 1/kRaceBlock of a per-entry race, and level 2 touches one
+// block.  Block variates use purpose SAMPLE (sub-index b / 4, word b % 4), entry
+// variates purpose SAMPLE_IN_BLOCK (sub-index v / 4, word v % 4).
+constexpr int kRaceBlock = 256;              // entries per block (one warp step: 32 lanes x 8)
+constexpr int kRaceQuad = 4 * kRaceBlock;    // the four blocks of one Philox call
+
+// Race variate of a Philox word: E = -ln(u), u = (2 * (word >> 9) + 1) * 2^-24.
+// With m = 2^24 * (1 - u), an odd integer below 2^24, E = -ln(1 - m * 2^-24).
 __device__ __forceinline__ uint32_t race_m(uint32_t word) { return ((word >> 8) & 0xFFFFFEu) ^ 0xFFFFFFu; }
 
-// One entry with weight w: key E / w.  The filter m < thr24 * w, thr24 =
-// 2^24 * (a key some lane of the warp already holds), skips the logarithm
-// when the entry cannot win (E >= 1 - u); a weight of 0 never passes it.
-// Entries arrive in increasing v per thread, so the strict comparison keeps
-// the lowest index on ties.
-__device__ __forceinline__ void race_entry(KeyState& best, float& thr24, float w, uint32_t m, int v) {
+// One race entry with weight w: key E / w.  The filter m < thr24 * w, thr24 =
+// 2^24 * (a key already held), skips the logarithm when the entry cannot win
+// (E >= 1 - u); a weight of 0 never passes it.  Entries arrive in increasing
+// index, so the strict comparison keeps the lowest index on ties.
+__device__ __forceinline__ void race_entry(KeyState& best, float& thr24, float w, uint32_t m, int idx) {
   const float mf = (float)m;
   if (mf < thr24 * w) {
     const float key = -log1pf(-(mf * 0x1p-24f)) / w;
     if (key < best.key) {
-      best = KeyState{key, v};
+      best = KeyState{key, idx};
       thr24 = fminf(thr24, key * 0x1p24f);
     }
   }
 }
 
-// After each group the warp shares its lowest key, so that an entry takes the
-// logarithm only if it could lead the whole warp (otherwise nearly every step
-// has some lane on the slow path).  Keys are >= 0 or +inf, so their bit
-// patterns order like unsigned integers.  Lanes whose chunk ended earlier have
-// left the loop; the reduction runs over the lanes still in it.
-__device__ __forceinline__ float warp_thr24(const KeyState& best) {
-  const unsigned act = __activemask();
-  return __uint_as_float(__reduce_min_sync(act, __float_as_uint(best.key))) * 0x1p24f;
+// Weight of entry v in the draw.  Residual: max(0, p - q) (normalised p);
+// Excl: p * S with the rejected one-hot draft z_excl removed; P: p * S.  The
+// roundings are explicit so that both levels compute identical weights.
+enum { kWeightResidual = 0, kWeightExcl = 1, kWeightP = 2 };
+template <int kMode>
+__device__ __forceinline__ float race_weight(float x, float qv, int v, float c2, float M2, float invS, int z_excl) {
+  const float ew = ex2_approx(__fmaf_rn(x, c2, -M2));  // p_v * S
+  if (kMode == kWeightResidual) return fmaxf(0.0f, __fsub_rn(__fmul_rn(ew, invS), qv));
+  if (kMode == kWeightExcl) return v == z_excl ? 0.0f : ew;
+  return ew;
 }
 
-// Race over [v0, v1) of the sampled row.  kGeneral: residual weights
-// max(0, p - q) into best_r.  Otherwise weights p * S (S the row's sum, which
-// does not change the argmin), the excluded draft token z_excl into best_p and
-// every other entry into best_r.
-// Vector form: 16-byte loads, groups of 8 entries (two Philox blocks) per
-// thread and step; needs v0, v1 multiples of 8 and aligned rows.  kShared:
-// row and qrow point at entry v0 of chunks staged in shared memory; otherwise
-// at entry 0 of the rows in global memory.
-template <typename T, typename Q, bool kGeneral, bool kShared = false>
-__device__ __forceinline__ void race_chunk_vec(const void* row, const void* qrow, int z_excl, int v0, int v1,
-                                               float c2, float M2, float invS, uint32_t position,
-                                               uint64_t req, uint32_t k0, uint32_t k1, KeyState& best_r,
-                                               KeyState& best_p) {
-  float thr24 = best_r.key * 0x1p24f;
-  for (int g8 = (v0 >> 3) + threadIdx.x; g8 * 8 < v1; g8 += kSampleThreads) {
-    float x[8], qv[8];
-    const int gi = kShared ? g8 - (v0 >> 3) : g8;
-    Row8<T>::template load<kShared>(row, gi, x);
-    if (kGeneral) Row8<Q>::template load<kShared>(qrow, gi, qv);
-    const uint4 r0 = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)(2 * g8)), k0, k1);
-    const uint4 r1 = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)(2 * g8 + 1)), k0, k1);
-    const uint32_t words[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+struct RaceArgs {
+  int z_excl;
+  float c2, M2, invS;
+  uint32_t position;
+  uint64_t req;
+  uint32_t k0, k1;
+};
+
+// Level 1 over quads [q_first, q_end) of the row, quad q to warp
+// (q - q_first) mod nwarps.  One warp step covers one block: lane l holds
+// entries 8l..8l+7 of it (kSrc 0: 16-byte loads from global memory, row at
+// entry 0; kSrc 1: the same from a chunk staged in shared memory that starts
+// at entry base_v) or entries l + 32e (kSrc 2: scalar loads, any layout).
+// Every lane computes the same block sum and so holds the same best block.
+enum { kSrcGlobalVec = 0, kSrcShared = 1, kSrcGlobalScalar = 2 };
+
+// Raw 16-byte words of lane l's 8 entries of the four blocks of quad q
+// (entries 1024q + 256s + 8l .. +7); blocks at or past V are not read.
+template <typename E, int kSrc>
+struct QuadWords {
+  static constexpr int kWords = sizeof(E) == 4 ? 2 : 1;  // 16-byte words per 8 entries
+  uint4 w[4][kWords];
+  __device__ __forceinline__ void load(const void* base, int q, int V, int base_v) {
+    const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const int v = g8 * 8 + e;
-      const float ew = ex2_approx(fmaf(x[e], c2, -M2));  // p_v * S
-      const uint32_t m = race_m(words[e]);
-      if (kGeneral) {
-        race_entry(best_r, thr24, fmaxf(0.0f, ew * invS - qv[e]), m, v);
-      } else if (v == z_excl) {
-        float own = best_p.key * 0x1p24f;
-        race_entry(best_p, own, ew, m, v);
-      } else {
-        race_entry(best_r, thr24, ew, m, v);
-      }
+    for (int s = 0; s < 4; ++s) {
+      const int v8 = q * kRaceQuad + s * kRaceBlock + 8 * lane;
+#pragma unroll
+      for (int h = 0; h < kWords; ++h)
+        w[s][h] = v8 < V ? load16<kSrc == kSrcShared>(static_cast<const uint4*>(base) + (((v8 - base_v) >> 3) * kWords + h))
+                         : make_uint4(0u, 0u, 0u, 0u);
     }
-    thr24 = fminf(thr24, warp_thr24(best_r));
   }
-}
+  __device__ __forceinline__ float get(int s, int e) const {
+    if (kWords == 2) {
+      const uint4& u = w[s][e >> 2];
+      const uint32_t x = (e & 3) == 0 ? u.x : (e & 3) == 1 ? u.y : (e & 3) == 2 ? u.z : u.w;
+      return __uint_as_float(x);
+    }
+    const uint4& u = w[s][0];
+    const uint32_t x = e < 2 ? u.x : e < 4 ? u.y : e < 6 ? u.z : u.w;
+    return (e & 1) ? bf16_hi(x) : bf16_lo(x);
+  }
+};
 
-// Scalar form of the same race (any alignment, any V): groups of 4 entries
-// (one Philox block) per thread and step.
-template <typename T, bool kGeneral>
-__device__ __forceinline__ void race_chunk_scalar(const T* row, const void* qrow, int q_dtype, int z_excl,
-                                                  int v0, int v1, float c2, float M2, float invS,
-                                                  uint32_t position, uint64_t req, uint32_t k0, uint32_t k1,
-                                                  KeyState& best_r, KeyState& best_p) {
-  float thr24 = best_r.key * 0x1p24f;
-  for (int grp = (v0 >> 2) + threadIdx.x; grp * 4 < v1; grp += kSampleThreads) {
-    const uint4 rnd = philox(draw_counter(position, req, SPEC_PURPOSE_SAMPLE, (uint32_t)grp), k0, k1);
-    const uint32_t words[4] = {rnd.x, rnd.y, rnd.z, rnd.w};
+// Level 1 over quads [q_first, q_end) of the row, quad q to warp
+// (q - q_first) mod nwarps.  One block is one warp step: lane l holds entries
+// 8l..8l+7 of it (kSrc 0: 16-byte loads from global memory, row at entry 0,
+// the whole quad's loads issued at once; kSrc 1: the same from a chunk staged
+// in shared memory that starts at entry base_v) or entries l + 32e (kSrc 2:
+// scalar loads, any layout).  Every lane computes the same block sum and so
+// holds the same best block.
+template <typename T, typename Q, int kMode, int kSrc>
+__device__ void race_level1(const void* row, const void* qrow, int q_dtype, int V, int base_v, int q_first,
+                            int q_end, int warp_id, int nwarps, const RaceArgs& a, KeyState& best) {
+  const int lane = threadIdx.x & 31;
+  float thr24 = best.key * 0x1p24f;
+  for (int q = q_first + warp_id; q < q_end; q += nwarps) {
+    if (kSrc == kSrcGlobalScalar) {
+      const uint4 r = philox(draw_counter(a.position, a.req, SPEC_PURPOSE_SAMPLE, (uint32_t)q), a.k0, a.k1);
+      const uint32_t words[4] = {r.x, r.y, r.z, r.w};
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int v = grp * 4 + e;
-      if (v < v0 || v >= v1) continue;
-      const float ew = ex2_approx(fmaf(load_elem(row + v), c2, -M2));  // p_v * S
-      const uint32_t m = race_m(words[e]);
-      if (kGeneral) {
-        race_entry(best_r, thr24, fmaxf(0.0f, ew * invS - load_any(qrow, q_dtype, v)), m, v);
-      } else if (v == z_excl) {
-        float own = best_p.key * 0x1p24f;
-        race_entry(best_p, own, ew, m, v);
-      } else {
-        race_entry(best_r, thr24, ew, m, v);
+      for (int s = 0; s < 4; ++s) {
+        const int vb = q * kRaceQuad + s * kRaceBlock;
+        float wsum = 0.0f;
+        if (vb < V) {
+          float x[8], qv[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int v = vb + lane + 32 * e;
+            x[e] = v < V ? load_elem(static_cast<const T*>(row) + v) : 0.0f;
+            qv[e] = (kMode == kWeightResidual && v < V) ? load_any(qrow, q_dtype, v) : 0.0f;
+          }
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int v = vb + lane + 32 * e;
+            if (v < V) wsum += race_weight<kMode>(x[e], qv[e], v, a.c2, a.M2, a.invS, a.z_excl);
+          }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xFFFFFFFFu, wsum, o);
+        race_entry(best, thr24, wsum, race_m(words[s]), 4 * q + s);
+      }
+    } else {
+      QuadWords<T, kSrc> xw;
+      QuadWords<Q, kSrc> qw;
+      xw.load(row, q, V, base_v);
+      if (kMode == kWeightResidual) qw.load(qrow, q, V, base_v);
+      const uint4 r = philox(draw_counter(a.position, a.req, SPEC_PURPOSE_SAMPLE, (uint32_t)q), a.k0, a.k1);
+      const uint32_t words[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+      for (int s = 0; s < 4; ++s) {
+        const int v8 = q * kRaceQuad + s * kRaceBlock + 8 * lane;
+        float wsum = 0.0f;
+        if (v8 < V) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            wsum += race_weight<kMode>(xw.get(s, e), kMode == kWeightResidual ? qw.get(s, e) : 0.0f, v8 + e, a.c2,
+                                       a.M2, a.invS, a.z_excl);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xFFFFFFFFu, wsum, o);
+        race_entry(best, thr24, wsum, race_m(words[s]), 4 * q + s);
       }
     }
-    thr24 = fminf(thr24, warp_thr24(best_r));
   }
 }
 
@@ -725,107 +777,95 @@ __device__ __forceinline__ KeyState cta_min_key(KeyState b, KeyState* sh) {
   return b;
 }
 
-// Dynamic shared memory of the sampling kernel: the logits chunk, then the q
-// chunk, each at a 128-byte boundary (16-byte loads path only).
-size_t sample_stage_bytes(const VerifyLaunch& p) {
-  if (!p.vec_s) return 0;
-  const size_t esize = p.logits_dtype == SPEC_F32 ? 4 : 2, qsize = p.q_dtype == SPEC_F32 ? 4 : 2;
-  const size_t lb = ((size_t)p.chunk_s * esize + 127) / 128 * 128;
-  return lb + (p.q ? (size_t)p.chunk_s * qsize : 0);
+// Level 2 in block b (one entry per thread; result in thread 0).
+template <typename T, int kMode>
+__device__ KeyState race_level2(const T* row, const void* qrow, int q_dtype, int V, int b, const RaceArgs& a,
+                                KeyState* sh) {
+  const int v = b * kRaceBlock + (int)threadIdx.x;
+  KeyState best{INFINITY, INT_MAX};
+  if (v < V) {
+    const float x = load_elem(row + v);
+    const float qv = kMode == kWeightResidual ? load_any(qrow, q_dtype, v) : 0.0f;
+    const float w = race_weight<kMode>(x, qv, v, a.c2, a.M2, a.invS, a.z_excl);
+    const uint4 r = philox(draw_counter(a.position, a.req, SPEC_PURPOSE_SAMPLE_IN_BLOCK, (uint32_t)(v >> 2)), a.k0,
+                           a.k1);
+    const uint32_t word = (v & 3) == 0 ? r.x : (v & 3) == 1 ? r.y : (v & 3) == 2 ? r.z : r.w;
+    if (w > 0.0f) best = KeyState{-log1pf(-((float)race_m(word) * 0x1p-24f)) / w, v};
+  }
+  return cta_min_key(best, sh);
+}
+
+// Level 1 of this CTA's part of the row, dispatched on the weight mode, the
+// q element type and the layout (16-byte loads need V % 8 == 0 and aligned
+// rows).
+template <typename T, int kMode>
+__device__ void race_level1_any(const VerifyLaunch& p, const void* row, const void* qrow, int q_first, int q_end,
+                                int warp_id, int nwarps, const RaceArgs& a, KeyState& best) {
+  if (p.vec_s) {
+    if (kMode == kWeightResidual && p.q_dtype == SPEC_F32)
+      race_level1<T, float, kMode, kSrcGlobalVec>(row, qrow, p.q_dtype, p.V, 0, q_first, q_end, warp_id, nwarps, a,
+                                                  best);
+    else
+      race_level1<T, __nv_bfloat16, kMode, kSrcGlobalVec>(row, qrow, p.q_dtype, p.V, 0, q_first, q_end, warp_id,
+                                                          nwarps, a, best);
+  } else {
+    race_level1<T, T, kMode, kSrcGlobalScalar>(row, qrow, p.q_dtype, p.V, 0, q_first, q_end, warp_id, nwarps, a,
+                                               best);
+  }
 }
 
 template <typename T>
 __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyLaunch p) {
-  extern __shared__ __align__(128) unsigned char stage[];
-  __shared__ uint64_t sh_bar;
+  __shared__ int sh_last, sh_b;
+  __shared__ KeyState sh_red[kSampleThreads / 32];
   const int i = blockIdx.x / p.NCS;
   const int cs = blockIdx.x - i * p.NCS;
   const int V = p.V;
+  const int warp = threadIdx.x >> 5;
   pdl_wait_prerequisites();  // the decisions of the streaming kernel
   const ReqRec rec = p.req_rec[i];
   if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
-  const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
-  const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
-  __shared__ int sh_last, sh_y;
-  __shared__ KeyState sh_red[kSampleThreads / 32];
 
-  // Residual race at a rejection with a drafter distribution q; otherwise the
-  // race on p (bonus row), or on p without the rejected one-hot draft.
-  const bool general_q = (rec.flags & 4) != 0;
+  RaceArgs ra;
+  ra.z_excl = rec.z_excl;
+  ra.c2 = p.c2;
+  ra.M2 = rec.M2;
+  ra.invS = rec.invS;
+  ra.position = rec.position;
+  ra.req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
+  const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+  ra.k0 = (uint32_t)seed;
+  ra.k1 = (uint32_t)(seed >> 32);
+  // Residual against a dense q at a rejection; p without the draft at a
+  // one-hot rejection; p at the bonus row.
+  const int mode = (rec.flags & 4) ? kWeightResidual : (rec.flags & 2) ? kWeightExcl : kWeightP;
   const T* row = static_cast<const T*>(p.logits) + (size_t)rec.srow * V;
   const size_t qsize = p.q_dtype == SPEC_F32 ? 4 : 2;
-  const void* qrow =
-      general_q ? (const void*)((const char*)p.q + ((size_t)i * p.K + rec.a) * (size_t)V * qsize) : nullptr;
-  const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
-  const float c2 = p.c2;
-  KeyState best_r{INFINITY, INT_MAX};
-  KeyState best_p{INFINITY, INT_MAX};  // one-hot rejection: the excluded draft
-  {
-    const int v0 = cs * p.chunk_s;
-    const int v1 = min(V, v0 + p.chunk_s);
-    if (p.stage_s) {
-      // Stage the chunk (and the q chunk) in shared memory with bulk copies:
-      // one round trip per CTA instead of one per group of 8 entries.
-      const uint32_t lbytes = (uint32_t)(v1 - v0) * (uint32_t)sizeof(T);
-      const uint32_t qbytes = general_q ? (uint32_t)(v1 - v0) * (uint32_t)qsize : 0u;
-      unsigned char* lstage = stage;
-      unsigned char* qstage = stage + ((size_t)p.chunk_s * sizeof(T) + 127) / 128 * 128;
-      if (threadIdx.x == 0) {
-        mbar_init(&sh_bar, 1);
-        mbar_init_fence();
-        mbar_arrive_tx(&sh_bar, lbytes + qbytes);
-        bulk_load(lstage, row + v0, lbytes, &sh_bar);
-        if (general_q) bulk_load(qstage, (const char*)qrow + (size_t)v0 * qsize, qbytes, &sh_bar);
-      }
-      __syncthreads();  // the barrier is initialised before anyone waits on it
-      if (!mbar_wait_bounded(&sh_bar, 0, kCopyWaitNs)) {
-        // The copy did not land: report it, give it a second bounded wait so
-        // that it does not write into a finished CTA, and skip the race.
-        if (threadIdx.x == 0) report(p.status, SPEC_ERR_TIMEOUT);
-        mbar_wait_bounded(&sh_bar, 0, kCopyWaitNs);
-      } else if (general_q) {
-        if (p.q_dtype == SPEC_F32)
-          race_chunk_vec<T, float, true, true>(lstage, qstage, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
-                                               rec.position, req, k0, k1, best_r, best_p);
-        else
-          race_chunk_vec<T, __nv_bfloat16, true, true>(lstage, qstage, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
-                                                       rec.position, req, k0, k1, best_r, best_p);
-      } else {
-        race_chunk_vec<T, T, false, true>(lstage, nullptr, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position,
-                                          req, k0, k1, best_r, best_p);
-      }
-    } else if (p.vec_s) {
-      if (general_q) {
-        if (p.q_dtype == SPEC_F32)
-          race_chunk_vec<T, float, true>(row, qrow, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position, req,
-                                         k0, k1, best_r, best_p);
-        else
-          race_chunk_vec<T, __nv_bfloat16, true>(row, qrow, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
-                                                 rec.position, req, k0, k1, best_r, best_p);
-      } else {
-        race_chunk_vec<T, T, false>(row, nullptr, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position, req,
-                                    k0, k1, best_r, best_p);
-      }
-    } else if (general_q) {
-      race_chunk_scalar<T, true>(row, qrow, p.q_dtype, rec.z_excl, v0, v1, c2, rec.M2, rec.invS, rec.position,
-                                 req, k0, k1, best_r, best_p);
-    } else {
-      race_chunk_scalar<T, false>(row, nullptr, p.q_dtype, rec.z_excl, v0, v1, c2, rec.M2, rec.invS,
-                                  rec.position, req, k0, k1, best_r, best_p);
-    }
-    // one-hot: the race on p is the residual race plus the excluded draft
-    if (!general_q && key_better(best_r, best_p)) best_p = best_r;
-  }
+  const void* qrow = mode == kWeightResidual
+                         ? (const void*)((const char*)p.q + ((size_t)i * p.K + rec.a) * (size_t)V * qsize)
+                         : nullptr;
 
-  // ---- CTA reduction; the last CTA of the request to arrive merges ----
-  best_r = cta_min_key(best_r, sh_red);
-  best_p = cta_min_key(best_p, sh_red);
+  // ---- level 1 over this CTA's chunk (whole quads) ----
+  const int v0 = cs * p.chunk_s;
+  const int v1 = min(V, v0 + p.chunk_s);
+  const int q_first = v0 / kRaceQuad;
+  const int q_end = (v1 + kRaceQuad - 1) / kRaceQuad;
+  KeyState best{INFINITY, INT_MAX};
+  if (mode == kWeightResidual)
+    race_level1_any<T, kWeightResidual>(p, row, qrow, q_first, q_end, warp, kSampleThreads / 32, ra, best);
+  else if (mode == kWeightExcl)
+    race_level1_any<T, kWeightExcl>(p, row, qrow, q_first, q_end, warp, kSampleThreads / 32, ra, best);
+  else
+    race_level1_any<T, kWeightP>(p, row, qrow, q_first, q_end, warp, kSampleThreads / 32, ra, best);
+
+  // ---- CTA reduction; the last CTA of the request to arrive goes on ----
+  best = cta_min_key(best, sh_red);
   if (threadIdx.x == 0) {
     RacePartial rp;
-    rp.key_r = best_r.key;
-    rp.idx_r = best_r.idx;
-    rp.key_p = best_p.key;
-    rp.idx_p = best_p.idx;
+    rp.key_r = best.key;
+    rp.idx_r = best.idx;
+    rp.key_p = INFINITY;
+    rp.idx_p = INT_MAX;
     p.race_part[(size_t)i * p.NCS + cs] = rp;
     __threadfence();
     sh_last = atomicAdd(p.counters + i, 1u) == (uint32_t)(p.NCS - 1);
@@ -834,44 +874,59 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   if (!sh_last) return;
 
   __threadfence();
-  if (threadIdx.x == 0) {
-    KeyState r_all{INFINITY, INT_MAX}, p_all{INFINITY, INT_MAX};
-    for (int k = 0; k < p.NCS; ++k) {
+  if (warp == 0) {
+    // the partials of all chunks at once, one lane each
+    const int lane = threadIdx.x & 31;
+    KeyState all{INFINITY, INT_MAX};
+    for (int k = lane; k < p.NCS; k += 32) {
       const RacePartial* src = p.race_part + (size_t)i * p.NCS + k;
       KeyState kr{__ldcg(&src->key_r), __ldcg(&src->idx_r)};
-      KeyState kp{__ldcg(&src->key_p), __ldcg(&src->idx_p)};
-      if (key_better(kr, r_all)) r_all = kr;
-      if (key_better(kp, p_all)) p_all = kp;
+      if (key_better(kr, all)) all = kr;
     }
-    p.counters[i] = 0u;  // leave the workspace zeroed for the next call
-    // bonus: race on p_n; one-hot rejection with an empty residual: race on p
-    sh_y = r_all.idx != INT_MAX ? r_all.idx : (general_q ? -2 : p_all.idx);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      KeyState other{__shfl_xor_sync(0xFFFFFFFFu, all.key, o), __shfl_xor_sync(0xFFFFFFFFu, all.idx, o)};
+      if (key_better(other, all)) all = other;
+    }
+    if (lane == 0) {
+      p.counters[i] = 0u;  // leave the workspace zeroed for the next call
+      sh_b = all.idx;
+    }
   }
   __syncthreads();
-  int y = sh_y;
-  if (y == -2) {
-    // Residual max(0, p - q) empty in fp32 (p <= q everywhere): draw from p.
-    // The whole row in this CTA; this happens only when p and q agree to
-    // rounding at a rejection.
-    KeyState bp{INFINITY, INT_MAX}, unused{INFINITY, INT_MAX};
-    if (p.vec_s)
-      race_chunk_vec<T, T, false>(row, nullptr, -1, 0, V, c2, rec.M2, rec.invS, rec.position, req, k0, k1, bp,
-                                  unused);
-    else
-      race_chunk_scalar<T, false>(row, nullptr, p.q_dtype, -1, 0, V, c2, rec.M2, rec.invS, rec.position, req, k0,
-                                  k1, bp, unused);
+  int b = sh_b;
+  int wmode = mode;
+  if (b == INT_MAX) {
+    // Every weight is zero: an empty residual (p <= q in fp32, or p all on
+    // the one-hot draft).  Draw from p instead, the whole row in this CTA.
+    wmode = kWeightP;
+    KeyState bp{INFINITY, INT_MAX};
+    race_level1_any<T, kWeightP>(p, row, nullptr, 0, (V + kRaceQuad - 1) / kRaceQuad, warp, kSampleThreads / 32,
+                                 ra, bp);
     bp = cta_min_key(bp, sh_red);
-    y = bp.idx;
+    if (threadIdx.x == 0) sh_b = bp.idx;
+    __syncthreads();
+    b = sh_b;
+  }
+  // ---- level 2 inside block b ----
+  KeyState y{INFINITY, INT_MAX};
+  if (b != INT_MAX) {
+    if (wmode == kWeightResidual)
+      y = race_level2<T, kWeightResidual>(row, qrow, p.q_dtype, V, b, ra, sh_red);
+    else if (wmode == kWeightExcl)
+      y = race_level2<T, kWeightExcl>(row, qrow, p.q_dtype, V, b, ra, sh_red);
+    else
+      y = race_level2<T, kWeightP>(row, qrow, p.q_dtype, V, b, ra, sh_red);
   }
   if (threadIdx.x != 0) return;
   int32_t* tok = p.out_tokens + (size_t)i * (p.K + 1);
-  if (y == INT_MAX) {
+  if (y.idx == INT_MAX) {
     report(p.status, SPEC_ERR_BAD_INPUT);
     tok[rec.a] = -1;
     p.accepted_len[i] = 0;
     return;
   }
-  tok[rec.a] = y;
+  tok[rec.a] = y.idx;
 }
 
 // ---------------------------------------------------------------------------
@@ -891,17 +946,12 @@ static cudaError_t launch_typed(const VerifyLaunch& p, cudaStream_t stream, cuda
   if (err != cudaSuccess) return err;
   if (ev_after) cudaEventRecord(ev_after, stream);
   if (greedy) return cudaSuccess;
-  const size_t smem = p.stage_s ? sample_stage_bytes(p) : 0;
-  if (smem > 48 * 1024) {
-    err = cudaFuncSetAttribute(sample_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (err != cudaSuccess) return err;
-  }
   // Programmatic dependent launch: the sampling CTAs are launched while the
   // streaming kernel drains and wait (griddepcontrol.wait) for its completion.
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)((long long)p.B * p.NCS));
   cfg.blockDim = dim3(kSampleThreads);
-  cfg.dynamicSmemBytes = smem;
+  cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

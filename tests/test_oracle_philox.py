@@ -76,9 +76,10 @@ def test_variates_follow_the_counter_layout():
                                  [_u32(seed), _u32(seed >> 32)])
         assert oracle.accept_uniform(seed, req, pos) == (int(w[0]) >> 8) / 2.0**24
         for v in [0, 1, 2, 3, 4, 4097, 201087]:
-            w = oracle.philox4x32_10([_u32(pos), _u32(req), _u32(req >> 32), (2 << 28) | (v >> 2)],
-                                     [_u32(seed), _u32(seed >> 32)])
-            assert oracle.race_exponential(seed, req, pos, v) == oracle.race_variate(int(w[v & 3]))
+            for level, purpose in [(1, 2), (2, 3)]:
+                w = oracle.philox4x32_10([_u32(pos), _u32(req), _u32(req >> 32), (purpose << 28) | (v >> 2)],
+                                         [_u32(seed), _u32(seed >> 32)])
+                assert oracle.race_exponential(seed, req, pos, v, level) == oracle.race_variate(int(w[v & 3]))
 
 
 def test_accept_uniform_is_uniform():
@@ -92,7 +93,7 @@ def test_accept_uniform_is_uniform():
 
 
 def test_race_exponentials_are_unit_exponential():
-    e = np.array([oracle.race_exponential(1, 2, 3, v) for v in range(1 << 16)])
+    e = np.array([oracle.race_exponential(1, 2, 3, v, 2) for v in range(1 << 16)])
     assert e.min() >= 0.0
     assert stats.kstest(e, "expon").pvalue > 1e-4
     # the four words of one block are independent of each other

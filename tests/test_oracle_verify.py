@@ -233,6 +233,45 @@ def test_one_hot_rejection_draws_target_without_the_draft():
     assert stats.chisquare(np.delete(counts, z), rej.sum() * np.delete(w / w.sum(), z)).pvalue > 1e-3
 
 
+def _draws(rows, drafts, q, t, N, chunk=20000):
+    """Outcomes of N requests that verify the same rows, seeds 0..N-1."""
+    acc, tok = [], []
+    for s0 in range(0, N, chunk):
+        m = min(chunk, N - s0)
+        res = oracle.verify_batch(np.tile(rows, (m, 1)), np.tile(drafts, (m, 1)),
+                                  None if q is None else np.tile(q[None], (m, 1, 1)), t,
+                                  np.arange(s0, s0 + m, dtype=np.uint64), np.zeros(m, np.uint64),
+                                  np.zeros(m, np.int64))
+        acc.append(res["accepted"])
+        tok.append(res["tokens"])
+    return np.concatenate(acc), np.concatenate(tok)
+
+
+def test_draws_span_several_race_blocks():
+    """V = 1100 spans five blocks of the two-level race (the last one partial):
+    the bonus draw follows p and the residual draw follows norm(max(0, p - q))."""
+    rng = np.random.default_rng(17)
+    V, t, N = 1100, 1.0, 200000
+    rows = rng.normal(0, 1.0, (2, V)).astype(np.float32)
+    # bonus: q <= p at the draft, so it is always accepted and row 1 is drawn
+    acc, tok = _draws(rows, np.array([[5]], np.int32), np.full((1, V), 1e-30, np.float32), t, N)
+    assert (acc == 1).all()
+    counts = np.bincount(tok[:, 1], minlength=V)
+    assert stats.chisquare(counts, N * _softmax64(rows[1], t)).pvalue > 1e-3
+    # residual: a draft distribution far from p, drafts drawn from it
+    qv = _softmax64(rows[0] + rng.normal(0, 2.0, V), 1.0).astype(np.float32)
+    p = _softmax64(rows[0], t)
+    z = int(np.argmax(qv.astype(np.float64) - p))                      # q(z) > p(z): often rejected
+    acc, tok = _draws(rows, np.array([[z]], np.int32), qv[None, :], t, N)
+    rej = acc == 0
+    resid = np.maximum(0.0, p - qv.astype(np.float64))
+    assert rej.mean() == pytest.approx(1.0 - min(1.0, p[z] / float(qv[z])), abs=5e-3)
+    counts = np.bincount(tok[rej, 0], minlength=V)
+    keep = resid > 0
+    assert counts[~keep].sum() == 0
+    assert stats.chisquare(counts[keep], rej.sum() * resid[keep] / resid.sum()).pvalue > 1e-3
+
+
 # ---------------------------------------------------------------------------
 # Determinism (replay gives the same bits) and bad inputs
 # ---------------------------------------------------------------------------
