@@ -36,7 +36,7 @@
 namespace spec {
 
 constexpr int kStreamThreads = 256;
-constexpr int kUnroll = 4;
+constexpr int kUnroll = 8;
 constexpr int kSampleThreads = 256;
 constexpr int kMaxRows = SPEC_MAX_DRAFTS + 1;
 
@@ -46,9 +46,10 @@ static inline long long round_up(long long a, long long b) { return ceil_div(a, 
 VerifyGeometry verify_geometry(int B, int K, int V) {
   VerifyGeometry g{};
   const long long R_max = (long long)B * (K + 1);
-  // Streaming pass: aim for ~4096 (row, chunk) items of >= 4096 elements.
+  // Streaming pass: aim for ~4096 (row, chunk) items of >= 16384 elements
+  // (two rounds of 8 16-byte loads per thread for bf16).
   long long nc = ceil_div(4096, R_max);
-  nc = std::max(1LL, std::min(nc, std::max(1LL, (long long)V / 4096)));
+  nc = std::max(1LL, std::min(nc, std::max(1LL, (long long)V / 16384)));
   long long chunk = round_up(ceil_div(V, nc), 8);
   nc = ceil_div(V, chunk);  // every chunk non-empty
   // Sampling pass: aim for ~560 (request, chunk) CTAs, about one resident
@@ -111,6 +112,12 @@ __device__ __forceinline__ bool key_better(KeyState a, KeyState b) {
   return a.key < b.key || (a.key == b.key && a.idx < b.idx);
 }
 
+// Barrier over the kStreamThreads threads that stream and decide (threads
+// 0..kStreamThreads-1; a producer warp beyond them does not take part).
+__device__ __forceinline__ void consumer_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kStreamThreads) : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // Decision chain (the last streaming CTA of a request)
 // ---------------------------------------------------------------------------
@@ -140,20 +147,40 @@ __device__ __forceinline__ ReqShape request_shape(const VerifyLaunch& p, int i) 
   return s;
 }
 
-// All threads of the CTA.  Merges the chunk partials of rows 0..n, tests
-// every kept draft, writes the committed prefix, and either the argmax token
-// (t = 0) or the record of the row to sample (t > 0).  The arithmetic is fp32:
-// p_j(z) = 2^(l_z*c2 - fl(m*c2)) / S carries a relative error of a few 1e-7,
-// inside the 1e-5 tolerance on probabilities, and an acceptance decision can
-// move only where |u - min(1, p/q)| is of that order.
+// One warp.  Merges the chunk partials of rows 0..n (a lane per row), tests
+// every kept draft (a lane per draft), writes the committed prefix, and either
+// the argmax token (t = 0) or the record of the row to sample (t > 0).  Only
+// one warp of a CTA decides at a time (its shared arrays are per CTA).  The
+// arithmetic is fp32: p_j(z) = 2^(l_z*c2 - fl(m*c2)) / S carries a relative
+// error of a few 1e-7, inside the 1e-5 tolerance on probabilities, and an
+// acceptance decision can move only where |u - min(1, p/q)| is of that order.
+// What a decision reads first (seeds and draft tokens), loaded by the
+// deciding warp before it learns whether it decides, so that these loads
+// overlap the arrival atomic.  z[u] is draft j = lane + 32u.
+struct DecidePre {
+  uint32_t pos;
+  unsigned long long seed, req;
+  int32_t z[(kMaxRows + 31) / 32];
+};
+__device__ __forceinline__ DecidePre decide_prefetch(const VerifyLaunch& p, int i) {
+  const int lane = threadIdx.x & 31;
+  DecidePre pre;
+  pre.pos = (uint32_t)__ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
+  pre.seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+  pre.req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
+#pragma unroll
+  for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
+    const int j = lane + 32 * u;
+    pre.z[u] = j < p.K ? __ldg(p.drafts + (size_t)i * p.K + j) : 0;
+  }
+  return pre;
+}
+
 template <typename T, bool kGreedy>
-__device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs) {
-  const int K = p.K, V = p.V;
+__device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre) {
+  const int K = p.K, V = p.V, NC = p.NC;
   const float c2 = p.c2;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  __shared__ int sh_bad, sh_first_reject;
-  __shared__ uint32_t sh_pos;
-  __shared__ unsigned long long sh_seed, sh_req;
+  const int lane = threadIdx.x & 31;
   __shared__ float sh_m[kMaxRows];
   __shared__ float sh_S[kMaxRows];
   __shared__ int32_t sh_g[kMaxRows];
@@ -162,147 +189,134 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
   const int n = rs.n;
   const long long row0 = rs.row0;
 
-  // ---- round trip 1: seeds and draft tokens ----
-  if (threadIdx.x == 0) {
-    sh_pos = (uint32_t)p.pos_base[i];
-    sh_seed = p.seeds[i];
-    sh_req = p.request_ids[i];
-    sh_bad = rs.valid ? 0 : 1;
-    sh_first_reject = n;
-  }
-  for (int j = threadIdx.x; j < K; j += kStreamThreads) sh_z[j] = p.drafts[(size_t)i * K + j];
-  __syncthreads();
+  // ---- seeds and draft tokens (prefetched) ----
+  const uint32_t pos = pre.pos;
+  const unsigned long long seed = pre.seed, req = pre.req;
+#pragma unroll
+  for (int u = 0; u < (kMaxRows + 31) / 32; ++u)
+    if (lane + 32 * u < K) sh_z[lane + 32 * u] = pre.z[u];
+  __syncwarp();
 
-  // ---- round trip 2: the row partials (one warp per row, up to four rows
-  // per warp in flight) and, per draft, the target logit and the draft
-  // probability at the drafted token ----
-  const int jd = threadIdx.x;  // this thread's draft, if jd < n
-  float lz = 0.0f, qz = 1.0f;
-  bool zbad = false;
-  if (rs.valid && jd < n) {
-    const int z = sh_z[jd];
-    if (z < 0 || z >= V) {
-      zbad = true;
-    } else if (!kGreedy) {
-      lz = load_elem(static_cast<const T*>(p.logits) + (size_t)(row0 + jd) * V + z);
-      if (p.q) qz = load_any(p.q, p.q_dtype, ((int64_t)i * K + jd) * (int64_t)V + z);
-    }
-  }
+  // ---- round trip 2: row partials (a lane per row) and, per draft, the
+  // target logit and the draft probability at the drafted token ----
+  int bad = rs.valid ? 0 : 1;
   if (rs.valid) {
-    constexpr int kWarps = kStreamThreads / 32, kInFlight = 4;
-    for (int jb = warp; jb <= n; jb += kWarps * kInFlight) {
-      RowPartial rp[kInFlight];
+    for (int j = lane; j <= n; j += 32) {
+      const RowPartial* part = p.row_part + (size_t)(row0 + j) * NC;
+      int32_t f = 0;
+      // kBatch partials in flight per lane
+      constexpr int kBatch = 8;
+      if (kGreedy) {
+        ArgState best{-INFINITY, INT_MAX};
+        for (int c0 = 0; c0 < NC; c0 += kBatch) {
+          RowPartial rb[kBatch];
 #pragma unroll
-      for (int u = 0; u < kInFlight; ++u) {
-        const int j = jb + u * kWarps;
-        rp[u] = RowPartial{-INFINITY, 0.0f, INT_MAX, 0};
-        if (j <= n && lane < p.NC) rp[u] = load_partial_cg(p.row_part + (size_t)(row0 + j) * p.NC + lane);
-      }
+          for (int u = 0; u < kBatch; ++u)
+            if (c0 + u < NC) rb[u] = load_partial_cg(part + c0 + u);
 #pragma unroll
-      for (int u = 0; u < kInFlight; ++u) {
-        const int j = jb + u * kWarps;
-        if (j > n) break;
-        const RowPartial* part = p.row_part + (size_t)(row0 + j) * p.NC;
-        int32_t f = rp[u].flags;
-        if (kGreedy) {
-          ArgState best{-INFINITY, INT_MAX};
-          if (lane < p.NC) best = ArgState{rp[u].m, rp[u].idx};
-          for (int cc = lane + 32; cc < p.NC; cc += 32) {
-            const RowPartial r2 = load_partial_cg(part + cc);
-            f |= r2.flags;
-            ArgState o{r2.m, r2.idx};
+          for (int u = 0; u < kBatch; ++u) {
+            if (c0 + u >= NC) break;
+            f |= rb[u].flags;
+            ArgState o{rb[u].m, rb[u].idx};
             if (arg_better(o, best)) best = o;
           }
+        }
+        sh_m[j] = best.v;
+        sh_g[j] = best.idx;
+        if (f || best.idx == INT_MAX) bad = 1;
+      } else {
+        SoftState all{-INFINITY, 0.0f};
+        for (int c0 = 0; c0 < NC; c0 += kBatch) {
+          RowPartial rb[kBatch];
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-            ArgState other{__shfl_xor_sync(0xFFFFFFFFu, best.v, o),
-                           __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
-            if (arg_better(other, best)) best = other;
-          }
-          f = __reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
-          if (lane == 0) {
-            sh_m[j] = best.v;
-            sh_g[j] = best.idx;
-            if (f || best.idx == INT_MAX) atomicOr(&sh_bad, 1);
-          }
-        } else {
-          float m = rp[u].m;
-          for (int cc = lane + 32; cc < p.NC; cc += 32) m = fmaxf(m, load_partial_cg(part + cc).m);
+          for (int u = 0; u < kBatch; ++u)
+            if (c0 + u < NC) rb[u] = load_partial_cg(part + c0 + u);
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-          const float M2 = m * c2;
-          float S = 0.0f;
-          if (rp[u].m != -INFINITY) S += rp[u].s * exp2f(rp[u].m * c2 - M2);
-          for (int cc = lane + 32; cc < p.NC; cc += 32) {
-            const RowPartial r2 = load_partial_cg(part + cc);
-            f |= r2.flags;
-            if (r2.m != -INFINITY) S += r2.s * exp2f(r2.m * c2 - M2);
+          for (int u = 0; u < kBatch; ++u) {
+            if (c0 + u >= NC) break;
+            f |= rb[u].flags;
+            all = soft_merge(all, SoftState{rb[u].m, rb[u].s}, c2);
           }
+        }
+        sh_m[j] = all.m;
+        sh_S[j] = all.s;
+        if (f || !(all.m > -INFINITY) || !(all.s > 0.0f) || !isfinite(all.s)) bad = 1;
+      }
+    }
+  }
+  float lz[(kMaxRows + 31) / 32], qz[(kMaxRows + 31) / 32];
+  if (!kGreedy && rs.valid) {
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xFFFFFFFFu, S, o);
-          f = __reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
-          if (lane == 0) {
-            sh_m[j] = m;
-            sh_S[j] = S;
-            if (f || !(m > -INFINITY) || !(S > 0.0f) || !isfinite(S)) atomicOr(&sh_bad, 1);
-          }
+    for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
+      const int j = lane + 32 * u;
+      lz[u] = 0.0f;
+      qz[u] = 1.0f;
+      if (j < n) {
+        const int z = sh_z[j];
+        if (z >= 0 && z < V) {
+          lz[u] = load_elem(static_cast<const T*>(p.logits) + (size_t)(row0 + j) * V + z);
+          if (p.q) qz[u] = load_any(p.q, p.q_dtype, ((int64_t)i * K + j) * (int64_t)V + z);
         }
       }
     }
   }
-  if (zbad) atomicOr(&sh_bad, 1);
-  __syncthreads();
+  for (int j = lane; j < n; j += 32)
+    if (sh_z[j] < 0 || sh_z[j] >= V) bad = 1;
+  bad = __any_sync(0xFFFFFFFFu, bad);
+  __syncwarp();
 
-  // ---- acceptance test of every kept draft (one thread per draft) ----
-  if (!sh_bad && jd < n) {
-    const int z = sh_z[jd];
-    bool reject;
-    if (kGreedy) {
-      reject = z != sh_g[jd];
-      sh_pz[jd] = reject ? 0.0f : 1.0f;
-    } else {
-      // l_z * c2 - fl(m * c2) with one rounding
-      const float pz = exp2f(fmaf(lz, c2, -(sh_m[jd] * c2))) / sh_S[jd];
-      const bool qbad = p.q && (!(qz >= 0.0f) || isinf(qz));
-      float r;
-      if (qz > 0.0f)
-        r = fminf(1.0f, pz / qz);
-      else
-        r = pz > 0.0f ? 1.0f : 0.0f;
-      const uint64_t seed = sh_seed;
-      const uint4 w = philox(draw_counter(sh_pos + (uint32_t)jd, sh_req, SPEC_PURPOSE_ACCEPT, 0u),
-                             (uint32_t)seed, (uint32_t)(seed >> 32));
-      const float u = (float)(w.x >> 8) * 0x1p-24f;  // exact
-      reject = !(u < r);
-      sh_pz[jd] = pz;
-      if (qbad) {
-        atomicOr(&sh_bad, 1);
-        reject = false;
+  // ---- acceptance test of every kept draft (a lane per draft) ----
+  int first_reject = n;
+  if (!bad) {
+#pragma unroll
+    for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
+      const int j = lane + 32 * u;
+      if (j >= n) break;
+      const int z = sh_z[j];
+      bool reject;
+      if (kGreedy) {
+        reject = z != sh_g[j];
+        sh_pz[j] = reject ? 0.0f : 1.0f;
+      } else {
+        // l_z * c2 - fl(m * c2) with one rounding
+        const float pz = exp2f(fmaf(lz[u], c2, -(sh_m[j] * c2))) / sh_S[j];
+        if (p.q && (!(qz[u] >= 0.0f) || isinf(qz[u]))) bad = 1;
+        float r;
+        if (qz[u] > 0.0f)
+          r = fminf(1.0f, pz / qz[u]);
+        else
+          r = pz > 0.0f ? 1.0f : 0.0f;
+        const uint4 w = philox(draw_counter(pos + (uint32_t)j, req, SPEC_PURPOSE_ACCEPT, 0u), (uint32_t)seed,
+                               (uint32_t)(seed >> 32));
+        const float uu = (float)(w.x >> 8) * 0x1p-24f;  // exact
+        reject = !(uu < r);
+        sh_pz[j] = pz;
       }
+      if (reject) first_reject = min(first_reject, j);
     }
-    if (reject) atomicMin(&sh_first_reject, jd);
   }
-  __syncthreads();
+  bad = __any_sync(0xFFFFFFFFu, bad);
+  first_reject = (int)__reduce_min_sync(0xFFFFFFFFu, (unsigned)first_reject);
+  __syncwarp();
 
-  const bool bad = sh_bad != 0;
-  const int a = bad ? 0 : sh_first_reject;
+  const int a = bad ? 0 : first_reject;
   int32_t* tok = p.out_tokens + (size_t)i * (K + 1);
   if (bad) {
-    if (threadIdx.x == 0) report(p.status, SPEC_ERR_BAD_INPUT);
-    for (int j = threadIdx.x; j <= K; j += kStreamThreads) tok[j] = -1;
-    if (threadIdx.x == 0) p.accepted_len[i] = 0;
+    if (lane == 0) report(p.status, SPEC_ERR_BAD_INPUT);
+    for (int j = lane; j <= K; j += 32) tok[j] = -1;
+    if (lane == 0) p.accepted_len[i] = 0;
     if (p.p_draft)
-      for (int j = threadIdx.x; j < K; j += kStreamThreads) p.p_draft[(size_t)i * K + j] = 0.0f;
+      for (int j = lane; j < K; j += 32) p.p_draft[(size_t)i * K + j] = 0.0f;
   } else {
-    for (int j = threadIdx.x; j <= K; j += kStreamThreads) {
+    for (int j = lane; j <= K; j += 32) {
       if (j < a) tok[j] = sh_z[j];
       else if (j > a) tok[j] = -1;
     }
-    if (threadIdx.x == 0) p.accepted_len[i] = a;
+    if (lane == 0) p.accepted_len[i] = a;
     if (p.p_draft)
-      for (int j = threadIdx.x; j < K; j += kStreamThreads) p.p_draft[(size_t)i * K + j] = j < n ? sh_pz[j] : 0.0f;
+      for (int j = lane; j < K; j += 32) p.p_draft[(size_t)i * K + j] = j < n ? sh_pz[j] : 0.0f;
     if (p.row_stats) {
-      for (int j = threadIdx.x; j <= n; j += kStreamThreads) {
+      for (int j = lane; j <= n; j += 32) {
         float2 st;
         if (kGreedy) {
           st = make_float2(sh_m[j], 0.0f);
@@ -316,7 +330,7 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
       }
     }
   }
-  if (threadIdx.x == 0) {
+  if (lane == 0) {
     if (kGreedy) {
       if (!bad) tok[a] = sh_g[a];
     } else {
@@ -324,7 +338,7 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
       rec.a = a;
       rec.flags = (bad ? 1 : 0) | (a < n ? 2 : 0) | (a < n && p.q != nullptr ? 4 : 0);
       rec.z_excl = (!bad && a < n) ? sh_z[a] : -1;
-      rec.position = sh_pos + (uint32_t)a;
+      rec.position = pos + (uint32_t)a;
       rec.srow = row0 + a;
       rec.M2 = bad ? 0.0f : sh_m[a] * c2;
       rec.invS = bad ? 0.0f : 1.0f / sh_S[a];
@@ -332,6 +346,7 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
     }
     p.req_count[i] = 0u;  // leave the workspace zeroed for the next call
   }
+  __syncwarp();
 }
 
 // ---------------------------------------------------------------------------
@@ -370,128 +385,131 @@ struct Vec<float> {
   }
 };
 
+// Per-thread state of a streamed chunk: softmax (m, s = sum 2^(l*c2 - fl(m*c2)))
+// at t > 0, lowest argmax at t = 0; flags bit 0 = NaN (or +inf at t > 0) seen.
+// At t = 0 the thread keeps the first 16-byte vector that holds its maximum
+// and locates the element inside it once, when the chunk ends (finalize).
 template <typename T, bool kGreedy>
-__global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const VerifyLaunch p) {
-  using VT = Vec<T>;
-  constexpr int VEC = VT::N;
-  const int per_req = (p.K + 1) * p.NC;
-  const int i = blockIdx.x / per_req;
-  const int rem = blockIdx.x - i * per_req;
-  const int j = rem / p.NC;
-  const int c = rem - j * p.NC;
-  const ReqShape rs = request_shape(p, i);
-  if (!(rs.valid ? j <= rs.n : (j == 0 && c == 0))) return;
-  // The sampling kernel may start launching once every CTA here has started;
-  // it waits for this grid's completion before it reads anything.
-  pdl_launch_dependents();
-  __shared__ int sh_last;
-  if (rs.valid) {
-    const long long r = rs.row0 + j;
-    const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.V;
-    const int v0 = c * p.chunk;
-    const int v1 = min(p.V, v0 + p.chunk);
-    const uintptr_t addr = reinterpret_cast<uintptr_t>(row + v0);
-    const int head = min((int)(((16u - (unsigned)(addr & 15u)) & 15u) / sizeof(T)), v1 - v0);
-    const int body0 = v0 + head;
-    const int nvec = (v1 - body0) / VEC;
-    const int tail0 = body0 + nvec * VEC;
-    const float c2 = p.c2;
+struct RowAcc {
+  int32_t flags = 0;
+  ArgState g{-INFINITY, INT_MAX};
+  SoftState st{-INFINITY, 0.0f};
+  float M2 = -INFINITY;    // fl(st.m * c2)
+  uint4 g_word{0u, 0u, 0u, 0u};  // t = 0: the vector holding the maximum ...
+  int g_v0 = INT_MAX;            // ... and the index of its first element
 
-    // thread state
-    int32_t flags = 0;
-    ArgState g{-INFINITY, INT_MAX};
-    SoftState st{-INFINITY, 0.0f};
-    float M2 = -INFINITY;  // fl(st.m * c2)
-
-    auto consume_scalar = [&](int v, float x) {
-      if (x != x) {
-        flags |= 1;
-        return;
+  __device__ __forceinline__ void scalar(int v, float x, float c2) {
+    if (x != x) {
+      flags |= 1;
+      return;
+    }
+    if (kGreedy) {
+      if (g.idx == INT_MAX || x > g.v) {  // a tie keeps the earlier element
+        g.v = x;
+        g.idx = v;
+        g_v0 = INT_MAX;
       }
-      if (kGreedy) {
-        if (g.idx == INT_MAX || x > g.v) {
-          g.v = x;
-          g.idx = v;
+    } else {
+      if (x == INFINITY) flags |= 1;
+      if (x > st.m) {
+        const float M2n = x * c2;
+        st.s = st.s * exp2f(M2 - M2n);
+        st.m = x;
+        M2 = M2n;
+      }
+      if (st.m != -INFINITY) st.s += ex2_approx(fmaf(x, c2, -M2));
+    }
+  }
+
+  // t = 0: resolve the kept vector into (max, lowest index); call once the
+  // thread's last element is in.
+  __device__ __forceinline__ void finalize() {
+    using VT = Vec<T>;
+    if (!kGreedy || g_v0 == INT_MAX) return;
+    int found = INT_MAX;
+#pragma unroll
+    for (int e = VT::N - 1; e >= 0; --e)
+      if (VT::get(g_word, e) == g.v) found = g_v0 + e;
+    g.idx = found;
+    g_v0 = INT_MAX;
+  }
+
+  // kN 16-byte vectors; vector u holds entries v_of[u] .., v_of[u] ==
+  // INT_MAX marks a padding vector (-inf entries), which adds nothing.
+  template <int kN>
+  __device__ __forceinline__ void tile(const uint4 (&w)[kN], const int (&v_of)[kN], float c2) {
+    using VT = Vec<T>;
+    constexpr int VEC = VT::N;
+    float wm[kN];
+    float tm = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < kN; ++u) {
+      wm[u] = VT::vmax(w[u]);
+      tm = fmax_nan(tm, wm[u]);
+    }
+    if (tm != tm) {
+      flags |= 1;
+      return;
+    }
+    if (kGreedy) {
+      // vectors arrive in increasing index order: the strict > keeps the
+      // first vector that reaches the maximum
+#pragma unroll
+      for (int u = 0; u < kN; ++u) {
+        if (v_of[u] != INT_MAX && (g.idx == INT_MAX || wm[u] > g.v)) {
+          g.v = wm[u];
+          g_word = w[u];
+          g_v0 = v_of[u];
+          g.idx = INT_MAX - 1;  // resolved by finalize()
         }
-      } else {
-        if (x == INFINITY) flags |= 1;
-        if (x > st.m) {
-          const float M2n = x * c2;
-          st.s = st.s * exp2f(M2 - M2n);
-          st.m = x;
-          M2 = M2n;
-        }
-        if (st.m != -INFINITY) st.s += ex2_approx(fmaf(x, c2, -M2));
       }
-    };
-
-    // head: elements before the first 16-byte boundary (lowest indices)
-    if ((int)threadIdx.x < head) consume_scalar(v0 + threadIdx.x, load_elem(row + v0 + threadIdx.x));
-
-    // body: 16-byte vectors, kUnroll vectors in flight per thread
-    const uint4* vp = reinterpret_cast<const uint4*>(row + body0);
-    for (int base = threadIdx.x; base < nvec; base += kStreamThreads * kUnroll) {
-      uint4 w[kUnroll];
-  #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int vi = base + u * kStreamThreads;
-        w[u] = vi < nvec ? ldg_stream(vp + vi) : make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad);
+    } else {
+      if (tm == INFINITY) flags |= 1;
+      if (tm > st.m) {
+        const float M2n = tm * c2;
+        st.s = st.s * exp2f(M2 - M2n);
+        st.m = tm;
+        M2 = M2n;
       }
-      float tm = VT::vmax(w[0]);
-  #pragma unroll
-      for (int u = 1; u < kUnroll; ++u) tm = fmax_nan(tm, VT::vmax(w[u]));
-      if (tm != tm) {
-        flags |= 1;
-        continue;
-      }
-      if (kGreedy) {
-        if (g.idx == INT_MAX || tm > g.v) {
-          // locate the first element equal to the tile max (index order)
-          int found = INT_MAX;
-  #pragma unroll
-          for (int u = 0; u < kUnroll; ++u) {
-  #pragma unroll
-            for (int e = 0; e < VEC; ++e) {
-              if (found == INT_MAX && VT::get(w[u], e) == tm)
-                found = body0 + (base + u * kStreamThreads) * VEC + e;
-            }
+      if (st.m != -INFINITY) {
+        // packed fp32 pairs: one FFMA2 and one FADD2 per two entries
+        const float2 c2v = make_float2(c2, c2), nM2 = make_float2(-M2, -M2);
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < kN; ++u) {
+#pragma unroll
+          for (int e = 0; e < VEC; e += 2) {
+            const float2 y = __ffma2_rn(make_float2(VT::get(w[u], e), VT::get(w[u], e + 1)), c2v, nM2);
+            const float2 ex = make_float2(ex2_approx(y.x), ex2_approx(y.y));
+            if ((e >> 1) & 1) acc1 = __fadd2_rn(acc1, ex);
+            else acc0 = __fadd2_rn(acc0, ex);
           }
-          g.v = tm;
-          g.idx = found;
         }
-      } else {
-        if (tm == INFINITY) flags |= 1;
-        if (tm > st.m) {
-          const float M2n = tm * c2;
-          st.s = st.s * exp2f(M2 - M2n);
-          st.m = tm;
-          M2 = M2n;
-        }
-        if (st.m != -INFINITY) {
-          float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  #pragma unroll
-          for (int u = 0; u < kUnroll; ++u) {
-  #pragma unroll
-            for (int e = 0; e < VEC; ++e) acc[e & 3] += ex2_approx(fmaf(VT::get(w[u], e), c2, -M2));
-          }
-          st.s += (acc[0] + acc[1]) + (acc[2] + acc[3]);
-        }
+        st.s += (acc0.x + acc0.y) + (acc1.x + acc1.y);
       }
     }
+  }
+};
 
-    // tail: the last < VEC elements (highest indices)
-    if (tail0 + (int)threadIdx.x < v1)
-      consume_scalar(tail0 + threadIdx.x, load_elem(row + tail0 + threadIdx.x));
-
-    // ---- CTA reduction ----
-    __shared__ float sh_a[kStreamThreads / 32];
-    __shared__ float sh_b[kStreamThreads / 32];
-    __shared__ int32_t sh_i[kStreamThreads / 32];
-    __shared__ int32_t sh_f[kStreamThreads / 32];
+// End of one (request, row, chunk) item, all threads of the CTA: the CTA
+// reduction and the chunk partial (valid requests), the arrival on the
+// request's counter, and the request's decision if this CTA arrived last.
+template <typename T, bool kGreedy>
+__device__ __forceinline__ void finish_item(const VerifyLaunch& p, RowAcc<T, kGreedy>& acc, int i, const ReqShape& rs,
+                                            long long r, int c) {
+  __shared__ float sh_a[kStreamThreads / 32];
+  __shared__ float sh_b[kStreamThreads / 32];
+  __shared__ int32_t sh_i[kStreamThreads / 32];
+  __shared__ int32_t sh_f[kStreamThreads / 32];
+  __shared__ int sh_last;
+  const float c2 = p.c2;
+  if (rs.valid) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    flags = __reduce_or_sync(0xFFFFFFFFu, (unsigned)flags);
+    acc.finalize();
+    const int32_t flags = __reduce_or_sync(0xFFFFFFFFu, (unsigned)acc.flags);
     if (kGreedy) {
-  #pragma unroll
+      ArgState g = acc.g;
+#pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         ArgState other{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
         if (arg_better(other, g)) g = other;
@@ -501,7 +519,7 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
         sh_i[warp] = g.idx;
         sh_f[warp] = flags;
       }
-      __syncthreads();
+      consumer_sync();
       if (threadIdx.x == 0) {
         ArgState best{sh_a[0], sh_i[0]};
         int32_t f = sh_f[0];
@@ -518,7 +536,8 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
         p.row_part[(size_t)r * p.NC + c] = out;
       }
     } else {
-  #pragma unroll
+      SoftState st = acc.st;
+#pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         SoftState other{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)};
         st = soft_merge(st, other, c2);
@@ -528,33 +547,94 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
         sh_b[warp] = st.s;
         sh_f[warp] = flags;
       }
-      __syncthreads();
+      consumer_sync();
       if (threadIdx.x == 0) {
-        SoftState acc{sh_a[0], sh_b[0]};
+        SoftState all{sh_a[0], sh_b[0]};
         int32_t f = sh_f[0];
         for (int k = 1; k < kStreamThreads / 32; ++k) {
-          acc = soft_merge(acc, SoftState{sh_a[k], sh_b[k]}, c2);
+          all = soft_merge(all, SoftState{sh_a[k], sh_b[k]}, c2);
           f |= sh_f[k];
         }
         RowPartial out;
-        out.m = acc.m;
-        out.s = acc.s;
+        out.m = all.m;
+        out.s = all.s;
         out.idx = 0;
         out.flags = f;
         p.row_part[(size_t)r * p.NC + c] = out;
       }
     }
   }
-  // ---- arrival; the last CTA of the request decides it ----
+  // ---- arrival; the last CTA of the request decides it (warp 0) ----
+  DecidePre pre;
+  if (threadIdx.x < 32) pre = decide_prefetch(p, i);
   if (threadIdx.x == 0) {
     __threadfence();  // the partial above before the count
     const uint32_t target = rs.valid ? (uint32_t)(rs.n + 1) * (uint32_t)p.NC : 1u;
     sh_last = atomicAdd(p.req_count + i, 1u) == target - 1u;
   }
-  __syncthreads();
-  if (!sh_last) return;
+  consumer_sync();
+  if (!sh_last || threadIdx.x >= 32) return;
   __threadfence();  // the other CTAs' partials after their counts
-  decide_request<T, kGreedy>(p, i, rs);
+  decide_request<T, kGreedy>(p, i, rs, pre);
+}
+
+// Item of CTA blockIdx.x: (request i, row j, chunk c), request-major, so
+// that the requests complete (and are decided) in order.
+struct StreamItem {
+  int i, j, c;
+};
+__device__ __forceinline__ StreamItem stream_item(const VerifyLaunch& p) {
+  const int per_req = (p.K + 1) * p.NC;
+  StreamItem it;
+  it.i = blockIdx.x / per_req;
+  const int rem = blockIdx.x - it.i * per_req;
+  it.j = rem / p.NC;
+  it.c = rem - it.j * p.NC;
+  return it;
+}
+
+// Streaming pass with 16-byte loads from global memory (any alignment: a
+// scalar head and tail around the aligned body).
+template <typename T, bool kGreedy>
+__global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const VerifyLaunch p) {
+  using VT = Vec<T>;
+  constexpr int VEC = VT::N;
+  const StreamItem it = stream_item(p);
+  const ReqShape rs = request_shape(p, it.i);
+  if (!(rs.valid ? it.j <= rs.n : (it.j == 0 && it.c == 0))) return;
+  // The sampling kernel may start launching once every CTA here has started;
+  // it waits for this grid's completion before it reads anything.
+  pdl_launch_dependents();
+  RowAcc<T, kGreedy> acc;
+  const long long r = rs.row0 + it.j;
+  if (rs.valid) {
+    const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.V;
+    const int v0 = it.c * p.chunk;
+    const int v1 = min(p.V, v0 + p.chunk);
+    const uintptr_t addr = reinterpret_cast<uintptr_t>(row + v0);
+    const int head = min((int)(((16u - (unsigned)(addr & 15u)) & 15u) / sizeof(T)), v1 - v0);
+    const int body0 = v0 + head;
+    const int nvec = (v1 - body0) / VEC;
+    const int tail0 = body0 + nvec * VEC;
+    // head: elements before the first 16-byte boundary (lowest indices)
+    if ((int)threadIdx.x < head) acc.scalar(v0 + threadIdx.x, load_elem(row + v0 + threadIdx.x), p.c2);
+    // body: 16-byte vectors, kUnroll vectors in flight per thread
+    const uint4* vp = reinterpret_cast<const uint4*>(row + body0);
+    for (int base = threadIdx.x; base < nvec; base += kStreamThreads * kUnroll) {
+      uint4 w[kUnroll];
+      int v_of[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int vi = base + u * kStreamThreads;
+        w[u] = vi < nvec ? ldg_stream(vp + vi) : make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad);
+        v_of[u] = vi < nvec ? body0 + vi * VEC : INT_MAX;
+      }
+      acc.template tile<kUnroll>(w, v_of, p.c2);
+    }
+    // tail: the last < VEC elements (highest indices)
+    if (tail0 + (int)threadIdx.x < v1) acc.scalar(tail0 + threadIdx.x, load_elem(row + tail0 + threadIdx.x), p.c2);
+  }
+  finish_item<T, kGreedy>(p, acc, it.i, rs, r, it.c);
 }
 
 // ---------------------------------------------------------------------------
@@ -825,6 +905,14 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   pdl_wait_prerequisites();  // the decisions of the streaming kernel
   const ReqRec rec = p.req_rec[i];
   if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
+  // The record comes from this call's decision when the workspace started
+  // zeroed; refuse one that could not (e.g. a workspace the caller did not
+  // leave as the library left it) rather than read outside the inputs.
+  if (rec.a < 0 || rec.a > p.K || rec.srow < 0 || rec.srow >= p.R_max || rec.z_excl < -1 || rec.z_excl >= V ||
+      ((rec.flags & 4) && (p.q == nullptr || rec.a >= p.K))) {
+    if (threadIdx.x == 0) report(p.status, SPEC_ERR_WORKSPACE);
+    return;
+  }
 
   RaceArgs ra;
   ra.z_excl = rec.z_excl;
