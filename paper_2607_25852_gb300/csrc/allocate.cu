@@ -101,6 +101,9 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
   __shared__ int sh_bad;
   const int tid = threadIdx.x;
   if (tid == 0) sh_bad = 0;
+  // The next kernel (the streaming pass) may launch now: it waits for this
+  // one's completion before it reads the depths and row offsets.
+  pdl_launch_dependents();
 
   // ---- every global input in one round trip, coalesced ----
   for (int q = tid; q < BK; q += kAllocThreads) {

@@ -25,6 +25,7 @@ __global__ void __launch_bounds__(kScanThreads) commit_scan_kernel(const CommitL
   __shared__ long long warp_tot[32];
   __shared__ long long carry;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  pdl_wait_prerequisites();  // accepted lengths come from the verification
   if (threadIdx.x == 0) carry = 0;
   __syncthreads();
   for (int base = 0; base < p.B; base += kScanThreads) {
@@ -62,6 +63,7 @@ __global__ void __launch_bounds__(kCommitThreads) commit_kernel(const CommitLaun
   const int K1 = p.K + 1;
   const int i = blockIdx.x / K1;
   const int j = blockIdx.x - i * K1;
+  pdl_wait_prerequisites();  // accepted lengths and tokens come from the verification
   const int a_raw = p.accepted_len[i];
   const int a = committed_len(p, i);
   if (j == 0 && threadIdx.x == 0 && a != a_raw) report(p.status, SPEC_ERR_BAD_INPUT);
@@ -116,14 +118,15 @@ __global__ void __launch_bounds__(kCommitThreads) commit_kernel(const CommitLaun
 
 cudaError_t launch_commit(const CommitLaunch& p, cudaStream_t stream) {
   const unsigned grid = (unsigned)((long long)p.B * (p.K + 1));
+  cudaError_t err;
   if (p.B <= kInlineScanMaxB) {
-    commit_kernel<false><<<grid, kCommitThreads, 0, stream>>>(p);
+    err = launch_after_previous(commit_kernel<false>, dim3(grid), dim3(kCommitThreads), 0, stream, p);
   } else {
-    commit_scan_kernel<<<1, kScanThreads, 0, stream>>>(p);
-    cudaError_t err = cudaGetLastError();
+    err = launch_after_previous(commit_scan_kernel, dim3(1), dim3(kScanThreads), 0, stream, p);
     if (err != cudaSuccess) return err;
-    commit_kernel<true><<<grid, kCommitThreads, 0, stream>>>(p);
+    err = launch_after_previous(commit_kernel<true>, dim3(grid), dim3(kCommitThreads), 0, stream, p);
   }
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 

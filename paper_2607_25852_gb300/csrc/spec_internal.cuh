@@ -81,6 +81,26 @@ __device__ __forceinline__ float load_any(const void* base, int dtype, int64_t i
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait_prerequisites() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// Launch `kernel` so that it may start while the previous kernel on the
+// stream drains (programmatic stream serialization).  Every kernel launched
+// this way calls pdl_wait_prerequisites() before it reads anything that an
+// earlier kernel writes, so the overlap covers launch latency only.
+template <typename... Args>
+inline cudaError_t launch_after_previous(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem,
+                                         cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // max with NaN propagation (PTX max.NaN)
 __device__ __forceinline__ float fmax_nan(float a, float b) {
   float d;

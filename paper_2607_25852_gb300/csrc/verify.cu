@@ -600,6 +600,7 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
   using VT = Vec<T>;
   constexpr int VEC = VT::N;
   const StreamItem it = stream_item(p);
+  pdl_wait_prerequisites();  // row offsets and depths come from the allocator
   const ReqShape rs = request_shape(p, it.i);
   if (!(rs.valid ? it.j <= rs.n : (it.j == 0 && it.c == 0))) return;
   // The sampling kernel may start launching once every CTA here has started;
@@ -903,6 +904,7 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   const int V = p.V;
   const int warp = threadIdx.x >> 5;
   pdl_wait_prerequisites();  // the decisions of the streaming kernel
+  pdl_launch_dependents();   // the commit kernel waits for this grid in turn
   const ReqRec rec = p.req_rec[i];
   if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
   // The record comes from this call's decision when the workspace started
@@ -1026,27 +1028,19 @@ static cudaError_t launch_typed(const VerifyLaunch& p, cudaStream_t stream, cuda
   const bool greedy = p.temperature == 0.0f;
   const unsigned grid1 = (unsigned)((long long)p.B * (p.K + 1) * p.NC);
   if (ev_before) cudaEventRecord(ev_before, stream);
-  if (greedy)
-    stream_rows_kernel<T, true><<<grid1, kStreamThreads, 0, stream>>>(p);
-  else
-    stream_rows_kernel<T, false><<<grid1, kStreamThreads, 0, stream>>>(p);
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = greedy ? launch_after_previous(stream_rows_kernel<T, true>, dim3(grid1), dim3(kStreamThreads), 0,
+                                                   stream, p)
+                           : launch_after_previous(stream_rows_kernel<T, false>, dim3(grid1), dim3(kStreamThreads),
+                                                   0, stream, p);
+  if (err != cudaSuccess) return err;
+  err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   if (ev_after) cudaEventRecord(ev_after, stream);
   if (greedy) return cudaSuccess;
-  // Programmatic dependent launch: the sampling CTAs are launched while the
-  // streaming kernel drains and wait (griddepcontrol.wait) for its completion.
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((unsigned)((long long)p.B * p.NCS));
-  cfg.blockDim = dim3(kSampleThreads);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, sample_kernel<T>, p);
+  // The sampling CTAs are launched while the streaming kernel drains and
+  // wait (griddepcontrol.wait) for its completion.
+  err = launch_after_previous(sample_kernel<T>, dim3((unsigned)((long long)p.B * p.NCS)), dim3(kSampleThreads), 0,
+                              stream, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
