@@ -61,7 +61,7 @@ extern "C" {
 typedef enum {
   SPEC_OK = 0,
   SPEC_ERR_INVALID_ARG = 1, /* host-visible argument error; nothing launched */
-  SPEC_ERR_WORKSPACE = 2,   /* workspace missing, too small or misaligned */
+  SPEC_ERR_WORKSPACE = 2,   /* workspace missing, too small or misaligned, or not left zeroed */
   SPEC_ERR_CUDA = 3,        /* a CUDA runtime call failed (e.g. launch) */
   SPEC_ERR_BAD_INPUT = 4,   /* device-detected data error (via *status) */
   SPEC_ERR_TIMEOUT = 5,     /* a bounded device wait gave up (via *status) */

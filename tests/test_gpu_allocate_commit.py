@@ -85,6 +85,19 @@ def test_random_allocations(B, K):
         assert_alloc_equal(g, r)
 
 
+def test_sixty_four_candidates():
+    """The most candidates a call takes (SPEC_MAX_CANDIDATES), with tied scores."""
+    rng = np.random.default_rng(64)
+    B, K = 256, 15
+    N = B * (K + 1)
+    conf = rng.choice([0.25, 0.5, 0.75, 1.0], size=(B, K)).astype(np.float32)
+    Ts = sorted(int(x) for x in rng.choice(np.arange(B, N + 1), size=64, replace=False))
+    costs = list(rng.uniform(0.5, 3.0, 64))
+    g = gpu_allocate(torch.as_tensor(conf), Ts, costs)
+    r = oracle.allocate(conf, Ts, costs)
+    assert_alloc_equal(g, r)
+
+
 def test_invalid_confidence_is_flagged():
     conf = torch.full((4, 3), 0.7)
     conf[2, 1] = float("nan")
