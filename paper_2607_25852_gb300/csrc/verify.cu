@@ -46,11 +46,12 @@ static inline long long round_up(long long a, long long b) { return ceil_div(a, 
 VerifyGeometry verify_geometry(int B, int K, int V) {
   VerifyGeometry g{};
   const long long R_max = (long long)B * (K + 1);
-  // Streaming pass: aim for ~4096 (row, chunk) items of >= 16384 elements
-  // (two rounds of 8 16-byte loads per thread for bf16).
+  // Streaming pass: aim for ~4096 (row, chunk) items, each a whole number of
+  // load rounds (256 threads x 8 16-byte vectors = 16384 bf16 entries), so
+  // that only the last chunk of a row ends in a partial round.
   long long nc = ceil_div(4096, R_max);
   nc = std::max(1LL, std::min(nc, std::max(1LL, (long long)V / 16384)));
-  long long chunk = round_up(ceil_div(V, nc), 8);
+  long long chunk = round_up(ceil_div(V, nc), 16384);
   nc = ceil_div(V, chunk);  // every chunk non-empty
   // Sampling pass: aim for ~560 (request, chunk) CTAs, about one resident
   // wave on 152 SMs, of >= 2048 elements each, every chunk a whole number of
@@ -112,8 +113,7 @@ __device__ __forceinline__ bool key_better(KeyState a, KeyState b) {
   return a.key < b.key || (a.key == b.key && a.idx < b.idx);
 }
 
-// Barrier over the kStreamThreads threads that stream and decide (threads
-// 0..kStreamThreads-1; a producer warp beyond them does not take part).
+// Barrier over the kStreamThreads threads of a streaming CTA.
 __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kStreamThreads) : "memory");
 }
@@ -147,13 +147,6 @@ __device__ __forceinline__ ReqShape request_shape(const VerifyLaunch& p, int i) 
   return s;
 }
 
-// One warp.  Merges the chunk partials of rows 0..n (a lane per row), tests
-// every kept draft (a lane per draft), writes the committed prefix, and either
-// the argmax token (t = 0) or the record of the row to sample (t > 0).  Only
-// one warp of a CTA decides at a time (its shared arrays are per CTA).  The
-// arithmetic is fp32: p_j(z) = 2^(l_z*c2 - fl(m*c2)) / S carries a relative
-// error of a few 1e-7, inside the 1e-5 tolerance on probabilities, and an
-// acceptance decision can move only where |u - min(1, p/q)| is of that order.
 // What a decision reads first (seeds and draft tokens), loaded by the
 // deciding warp before it learns whether it decides, so that these loads
 // overlap the arrival atomic.  z[u] is draft j = lane + 32u.
@@ -176,6 +169,13 @@ __device__ __forceinline__ DecidePre decide_prefetch(const VerifyLaunch& p, int 
   return pre;
 }
 
+// One warp.  Merges the chunk partials of rows 0..n (a lane per row), tests
+// every kept draft (a lane per draft), writes the committed prefix, and either
+// the argmax token (t = 0) or the record of the row to sample (t > 0).  Only
+// one warp of a CTA decides at a time (its shared arrays are per CTA).  The
+// arithmetic is fp32: p_j(z) = 2^(l_z*c2 - fl(m*c2)) / S carries a relative
+// error of a few 1e-7, inside the 1e-5 tolerance on probabilities, and an
+// acceptance decision can move only where |u - min(1, p/q)| is of that order.
 template <typename T, bool kGreedy>
 __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre) {
   const int K = p.K, V = p.V, NC = p.NC;
