@@ -64,8 +64,16 @@ __global__ void __launch_bounds__(kCommitThreads) commit_kernel(const CommitLaun
   const int i = blockIdx.x / K1;
   const int j = blockIdx.x - i * K1;
   pdl_wait_prerequisites();  // accepted lengths and tokens come from the verification
+  // ---- one round trip: this request's length and row, every length before
+  // it (inline offsets), and the token ----
   const int a_raw = p.accepted_len[i];
-  const int a = committed_len(p, i);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int before = 0;
+  if (!kScanned && (int)threadIdx.x < i) before = committed_len(p, threadIdx.x) + 1;
+  const long long row_i = p.row_offsets ? (long long)p.row_offsets[i] : (long long)i * K1;
+  const long long R = p.row_offsets ? (long long)p.row_offsets[p.B] : (long long)p.B * K1;
+  const int32_t token = threadIdx.x == 0 ? p.out_tokens[(size_t)i * K1 + j] : 0;
+  const int a = (a_raw >= 0 && a_raw <= p.K) ? a_raw : 0;  // out-of-range lengths count as 0 (reported)
   if (j == 0 && threadIdx.x == 0 && a != a_raw) report(p.status, SPEC_ERR_BAD_INPUT);
   if (j > a) return;
 
@@ -74,9 +82,8 @@ __global__ void __launch_bounds__(kCommitThreads) commit_kernel(const CommitLaun
     if (threadIdx.x == 0) sh_off = p.commit_offsets_out[i];
   } else {
     // sum_{i' < i} (a_{i'} + 1); i < kInlineScanMaxB <= kCommitThreads
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     __shared__ int warp_sum[kCommitThreads / 32];
-    int x = (int)threadIdx.x < i ? committed_len(p, threadIdx.x) + 1 : 0;
+    int x = before;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
     if (lane == 0) warp_sum[warp] = x;
@@ -93,11 +100,10 @@ __global__ void __launch_bounds__(kCommitThreads) commit_kernel(const CommitLaun
   }
   __syncthreads();
   const int dst = sh_off + j;
-  if (threadIdx.x == 0) p.packed_tokens_out[dst] = p.out_tokens[(size_t)i * K1 + j];
+  if (threadIdx.x == 0) p.packed_tokens_out[dst] = token;
   if (p.hidden == nullptr || p.hidden_out == nullptr) return;
 
-  const long long src_row = (p.row_offsets ? (long long)p.row_offsets[i] : (long long)i * K1) + j;
-  const long long R = p.row_offsets ? (long long)p.row_offsets[p.B] : (long long)p.B * K1;
+  const long long src_row = row_i + j;
   if (src_row < 0 || src_row >= R) {
     if (threadIdx.x == 0) report(p.status, SPEC_ERR_BAD_INPUT);
     return;
