@@ -75,6 +75,12 @@ def dist_init(world, backend):
     return dist
 
 
+def job_throughput(world, rows_per_rank, steps, total_ms):
+    """Whole-job verified positions/s: every rank verifies rows_per_rank rows
+    per step (weak scaling), timed as the slowest rank's total_ms."""
+    return world * rows_per_rank * steps / (total_ms * 1e-3)
+
+
 def max_over_ranks(dist, value, device):
     if dist is None:
         return value
@@ -399,7 +405,7 @@ def run_ours(args):
     step_ms = [a.elapsed_time(b) for a, b in ev]
     kern_ms = [a.elapsed_time(b) for a, b in kev]
     ms_per_step = total_ms / args.steps
-    value = world * R * args.steps / (total_ms * 1e-3)
+    value = job_throughput(world, R, args.steps, total_ms)
 
     # ---- end to end through the same API with pinned host buffers ----
     e2e = None
