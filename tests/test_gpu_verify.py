@@ -175,3 +175,38 @@ def test_argument_errors_raise():
             run_verify(wl.logits, wl.drafts, None, wl.B, wl.K, wl.V, t, wl.seeds, wl.request_ids,
                        wl.pos_base)
         assert e.value.code == spec.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("t", [0.0, 1.0])
+@pytest.mark.parametrize("qmode", ["onehot", "dense"])
+def test_most_drafts_per_request(t, qmode):
+    """K = SPEC_MAX_DRAFTS = 255: the decision's per-lane loops over 256 rows."""
+    wl = _random_case(600, "bf16", t, qmode, B=2, K=255, seed=5)
+    _check(wl, t)
+
+
+def test_many_requests():
+    """B = 512, K = 15: 8192 rows, the most the allocator takes; one chunk per row."""
+    wl = _random_case(2048, "bf16", 1.0, "dense", B=512, K=15, seed=6)
+    _check(wl, 1.0)
+
+
+@pytest.mark.parametrize("t", [0.0, 1.0])
+def test_misaligned_logits_and_q(t):
+    """Row bases 2 bytes off a 16-byte boundary: the streaming pass takes its
+    scalar head and tail, the sampling pass its scalar loads."""
+    wl = _random_case(4096, "bf16", t, "dense", B=4, K=5, seed=7)
+    dev = torch.device("cuda")
+
+    def shifted(x):
+        buf = torch.empty(x.numel() + 1, dtype=x.dtype, device=dev)
+        view = buf[1:].view(x.shape)
+        view.copy_(x.to(dev))
+        assert view.data_ptr() % 16 == 2
+        return view
+
+    logits, q = shifted(wl.logits), shifted(wl.q)
+    gpu = run_verify(logits, wl.drafts, q, wl.B, wl.K, wl.V, t, wl.seeds, wl.request_ids, wl.pos_base)
+    ref = run_oracle(wl.logits, wl.drafts, wl.q, t, wl.seeds, wl.request_ids, wl.pos_base)
+    assert gpu["status"] == 0 and (ref["status"] == 0).all()
+    compare(gpu, ref, wl.K, t)
