@@ -248,7 +248,7 @@ def measured_peak():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for name in ("verify.cu", "spec_internal.cuh"):
+    for name in ("verify.cu", "verify_common.cuh", "spec_internal.cuh"):
         with open(os.path.join(ROOT, "paper_2607_25852_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]

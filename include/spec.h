@@ -257,6 +257,101 @@ int spec_commit(const int32_t* accepted_len, const int32_t* out_tokens,
                 cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Vocabulary-sharded verification -- spec_verify for a target whose output
+ * layer is split over S tensor-parallel ranks (the paper serves its target
+ * with TP = 8, Section 4.4), each holding the logits (and q) of a contiguous
+ * column range [v_begin, v_begin + V_shard) of the vocabulary.  The ranges
+ * must cover [0, V) exactly once, in rank order; boundaries are arbitrary
+ * (201088 / 8 = 25136 columns per rank, say).  One round:
+ *   1. every rank: spec_shard_stats -> its stats records [R] (R = B(K+1));
+ *   2. all-gather the S ranks' records in shard order -> [S, R] records;
+ *   3. every rank: spec_shard_decide (identical results on every rank);
+ *   4. t > 0, every rank: spec_shard_sample -> its race records [B];
+ *   5. t > 0: all-gather them in shard order -> [S, B] records;
+ *   6. t > 0, every rank: spec_shard_finish writes the sampled tokens.
+ * The caller makes the two exchanges (all-gathers of S * R * 32 and
+ * S * B * 96 bytes; with every shard on one GPU, the records are simply
+ * written side by side).  The random variates are spec_verify's: they depend
+ * on vocabulary indices only, and a race block that straddles a shard
+ * boundary is completed in spec_shard_finish from the two shards' parts.
+ * Results: at t == 0 identical to spec_verify's bit for bit; at t > 0 the
+ * shard sums merge in another order than spec_verify's chunks, so
+ * probabilities agree within a few fp32 ulps and an acceptance or draw can
+ * differ only where its uniform or race keys tie to that precision.
+ * Records are opaque, 16-byte aligned device buffers of the sizes below.
+ * ---------------------------------------------------------------------- */
+#define SPEC_SHARD_STAT_BYTES 32     /* per (shard, packed row) */
+#define SPEC_SHARD_DECISION_BYTES 32 /* per request */
+#define SPEC_SHARD_RACE_BYTES 96     /* per (shard, request) */
+
+/* Workspace of spec_shard_stats and spec_shard_sample on one rank: 256-byte
+ * aligned, zero-filled once before its first use, left zeroed by every call;
+ * calls that may overlap on the device need separate workspaces.  0 for an
+ * invalid shape. */
+size_t spec_shard_workspace(int B, int K, int V_shard);
+
+/* spec_shard_stats -- per packed row, over the shard's columns: (max, sum of
+ * exp2(l * c2 - fl(max * c2))) at t > 0 with c2 = log2(e) / t, (max, lowest
+ * argmax as a vocabulary index) at t == 0; and, when the row's draft token
+ * falls in the shard, its logit and q value there.
+ *   logits_shard    device [R, V_shard] of logits_dtype (the shard's columns
+ *                   of the rows spec_verify takes), any alignment.
+ *   q_shard         device [B, K, V_shard] of q_dtype, or NULL (one-hot q).
+ *   row_offsets, depth, draft_tokens, pos_base, temperature, status: as
+ *                   spec_verify.
+ *   V               the whole vocabulary; v_begin, V_shard this shard's range.
+ *   stats_out       device [R] records of SPEC_SHARD_STAT_BYTES.
+ * Rows of requests whose depth or offsets are inconsistent are not written
+ * (spec_shard_decide reports them).  Returns SPEC_OK, SPEC_ERR_INVALID_ARG,
+ * SPEC_ERR_WORKSPACE or SPEC_ERR_CUDA. */
+int spec_shard_stats(const void* logits_shard, int logits_dtype, const int32_t* row_offsets,
+                     const int32_t* depth, const int32_t* draft_tokens, const void* q_shard,
+                     int q_dtype, int B, int K, int V, int v_begin, int V_shard,
+                     float temperature, const int64_t* pos_base, void* stats_out,
+                     int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* spec_shard_decide -- merges the S shards' records of each row (in shard
+ * order) and runs spec_verify's decision chain: accepted_len_out, out_tokens
+ * (all but the sampled token at t > 0), p_draft_out and row_stats_out as
+ * spec_verify writes them.
+ *   stats           device [S, R] records gathered from spec_shard_stats.
+ *   q_dense         nonzero if the ranks passed q_shard (t > 0).
+ *   decisions_out   device [B] records of SPEC_SHARD_DECISION_BYTES; required
+ *                   at t > 0, unused at t == 0 (may be NULL).
+ * A draft token owned by no shard, or by several, sets SPEC_ERR_BAD_INPUT for
+ * its request. */
+int spec_shard_decide(const void* stats, int S, const int32_t* row_offsets,
+                      const int32_t* depth, const int32_t* draft_tokens, int q_dense, int B,
+                      int K, int V, float temperature, const uint64_t* seeds,
+                      const uint64_t* request_ids, const int64_t* pos_base,
+                      int32_t* accepted_len_out, int32_t* out_tokens, float* p_draft_out,
+                      float* row_stats_out, void* decisions_out, int32_t* status,
+                      cudaStream_t stream);
+
+/* spec_shard_sample -- t > 0: level 1 of the draw over the race blocks the
+ * shard owns whole (with the race over p beside it at a rejection, for the
+ * case that no shard has a positive draw weight) and level 2 inside the best
+ * of them; for a block cut by a shard boundary, the shard's part of its
+ * weight sum and its part's best entry.  Does nothing at t == 0.
+ *   decisions       device [B] records from spec_shard_decide.
+ *   race_out        device [B] records of SPEC_SHARD_RACE_BYTES. */
+int spec_shard_sample(const void* logits_shard, int logits_dtype, const void* q_shard,
+                      int q_dtype, const void* decisions, int B, int K, int V, int v_begin,
+                      int V_shard, float temperature, const uint64_t* seeds,
+                      const uint64_t* request_ids, void* race_out, int32_t* status, void* ws,
+                      size_t ws_bytes, cudaStream_t stream);
+
+/* spec_shard_finish -- t > 0: completes the cut blocks (weight sums added in
+ * shard order, block variates drawn) and takes the lowest block key over all
+ * shards: each request's sampled token in out_tokens.  Does nothing at
+ * t == 0.
+ *   races           device [S, B] records gathered from spec_shard_sample. */
+int spec_shard_finish(const void* races, int S, const void* decisions, int B, int K, int V,
+                      float temperature, const uint64_t* seeds, const uint64_t* request_ids,
+                      int32_t* accepted_len_out, int32_t* out_tokens, int32_t* status,
+                      cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * spec_profile_stream_pass -- measurement aid.  The next spec_verify call
  * records `before` immediately before and `after` immediately after its
  * vocabulary-streaming kernel, on its stream, then forgets both.  Arguments

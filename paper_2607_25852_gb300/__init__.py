@@ -30,10 +30,16 @@ MAX_DRAFTS = 255
 MAX_ALLOC_POSITIONS = 8192
 MAX_CANDIDATES = 64
 
+SHARD_STAT_BYTES = 32
+SHARD_DECISION_BYTES = 32
+SHARD_RACE_BYTES = 96
+
 __all__ = [
     "SpecError", "spec_version", "spec_error_string", "spec_budget_from_ratios",
     "spec_allocate_workspace", "spec_allocate", "spec_verify_workspace", "spec_verify",
     "spec_verify_static", "spec_commit", "spec_profile_stream_pass", "verify_workspace", "library",
+    "spec_shard_workspace", "spec_shard_stats", "spec_shard_decide", "spec_shard_sample",
+    "spec_shard_finish", "shard_workspace",
 ]
 
 
@@ -164,6 +170,74 @@ def spec_commit(accepted_len, out_tokens, hidden, B, K, packed_tokens_out, commi
         B, K, H, _ptr(packed_tokens_out), _ptr(commit_offsets_out), _ptr(hidden_out),
         _ptr(status), _stream(stream))
     _check(code, "spec_commit")
+
+
+def spec_shard_workspace(B: int, K: int, V_shard: int) -> int:
+    return library().spec_shard_workspace(B, K, V_shard)
+
+
+def shard_workspace(B: int, K: int, V_shard: int, device="cuda"):
+    """A zero-filled workspace for spec_shard_stats / spec_shard_sample."""
+    n = spec_shard_workspace(B, K, V_shard)
+    if n == 0:
+        raise SpecError(ERR_INVALID_ARG, "spec_shard_workspace")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def _nbytes(t):
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def spec_shard_stats(logits_shard, draft_tokens, q_shard, B, K, V, v_begin, temperature, pos_base,
+                     stats_out, ws, row_offsets=None, depth=None, status=None, stream=None):
+    """logits_shard [R, V_shard]; q_shard [B, K, V_shard] or None; stats_out >= R * 32 bytes."""
+    R = B * (K + 1)
+    if _nbytes(stats_out) < R * SHARD_STAT_BYTES:
+        raise SpecError(ERR_INVALID_ARG, "spec_shard_stats: stats_out too small")
+    code = library().spec_shard_stats(
+        _ptr(logits_shard), _dtype(logits_shard), _ptr(row_offsets), _ptr(depth), _ptr(draft_tokens),
+        _ptr(q_shard), _dtype(q_shard), B, K, V, v_begin, logits_shard.shape[-1], float(temperature),
+        _ptr(pos_base), _ptr(stats_out), _ptr(status), _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(code, "spec_shard_stats")
+
+
+def spec_shard_decide(stats, S, draft_tokens, q_dense, B, K, V, temperature, seeds, request_ids,
+                      pos_base, accepted_len_out, out_tokens, decisions_out=None, row_offsets=None,
+                      depth=None, p_draft_out=None, row_stats_out=None, status=None, stream=None):
+    """stats: the S shards' records [S, B(K+1)] (>= S * B(K+1) * 32 bytes)."""
+    if _nbytes(stats) < S * B * (K + 1) * SHARD_STAT_BYTES:
+        raise SpecError(ERR_INVALID_ARG, "spec_shard_decide: stats too small")
+    if decisions_out is not None and _nbytes(decisions_out) < B * SHARD_DECISION_BYTES:
+        raise SpecError(ERR_INVALID_ARG, "spec_shard_decide: decisions_out too small")
+    code = library().spec_shard_decide(
+        _ptr(stats), S, _ptr(row_offsets), _ptr(depth), _ptr(draft_tokens), int(bool(q_dense)), B, K, V,
+        float(temperature), _ptr(seeds), _ptr(request_ids), _ptr(pos_base), _ptr(accepted_len_out),
+        _ptr(out_tokens), _ptr(p_draft_out), _ptr(row_stats_out), _ptr(decisions_out), _ptr(status),
+        _stream(stream))
+    _check(code, "spec_shard_decide")
+
+
+def spec_shard_sample(logits_shard, q_shard, decisions, B, K, V, v_begin, temperature, seeds,
+                      request_ids, race_out, ws, status=None, stream=None):
+    """race_out >= B * 96 bytes."""
+    if _nbytes(race_out) < B * SHARD_RACE_BYTES or _nbytes(decisions) < B * SHARD_DECISION_BYTES:
+        raise SpecError(ERR_INVALID_ARG, "spec_shard_sample: record buffer too small")
+    code = library().spec_shard_sample(
+        _ptr(logits_shard), _dtype(logits_shard), _ptr(q_shard), _dtype(q_shard), _ptr(decisions), B, K,
+        V, v_begin, logits_shard.shape[-1], float(temperature), _ptr(seeds), _ptr(request_ids),
+        _ptr(race_out), _ptr(status), _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(code, "spec_shard_sample")
+
+
+def spec_shard_finish(races, S, decisions, B, K, V, temperature, seeds, request_ids,
+                      accepted_len_out, out_tokens, status=None, stream=None):
+    """races: the S shards' race records [S, B] (>= S * B * 96 bytes)."""
+    if _nbytes(races) < S * B * SHARD_RACE_BYTES or _nbytes(decisions) < B * SHARD_DECISION_BYTES:
+        raise SpecError(ERR_INVALID_ARG, "spec_shard_finish: record buffer too small")
+    code = library().spec_shard_finish(
+        _ptr(races), S, _ptr(decisions), B, K, V, float(temperature), _ptr(seeds), _ptr(request_ids),
+        _ptr(accepted_len_out), _ptr(out_tokens), _ptr(status), _stream(stream))
+    _check(code, "spec_shard_finish")
 
 
 def spec_profile_stream_pass(before=None, after=None):

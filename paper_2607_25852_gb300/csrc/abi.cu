@@ -143,6 +143,7 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
   p.depth = depth;
   p.drafts = draft_tokens;
   p.q = temperature > 0.0f ? q : nullptr;
+  p.dense_q = p.q != nullptr;
   p.q_dtype = q_dtype;
   p.B = B;
   p.K = K;

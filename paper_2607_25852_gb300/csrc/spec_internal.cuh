@@ -169,6 +169,7 @@ struct VerifyLaunch {
   const int32_t* drafts;
   const void* q;
   int q_dtype;
+  bool dense_q;         // q given (t > 0): residual draws against it
   int B, K, V;
   float temperature;
   float c2;            // log2(e) / t  (0 when t == 0)

@@ -112,3 +112,54 @@ def compare(gpu, ref, K, t, depth=None, row_offsets=None, check_stats=True):
         np.testing.assert_allclose(gpu["row_stats"][rows, 1], ref["row_logS"][rows], rtol=0, atol=P_RTOL)
     assert n_acc_ties + n_race_ties <= max(1, 1e-4 * positions), (n_acc_ties, n_race_ties, positions)
     return n_acc_ties, n_race_ties, positions
+
+
+def shard_bounds(V, S, unit=1):
+    """S contiguous ranges covering [0, V): equal parts rounded to `unit`
+    columns, the last one taking the rest."""
+    per = max(unit, (V // S) // unit * unit)
+    b = [min(V, s * per) for s in range(S)] + [V]
+    return b
+
+
+def run_sharded(logits, drafts, q, B, K, V, t, seeds, request_ids, pos_base, bounds,
+                row_offsets=None, depth=None, ws=None, device="cuda"):
+    """The four shard calls over shards [bounds[s], bounds[s+1]) of one GPU;
+    the records of the S shards are written side by side (the exchange).
+    `ws`: the per-shard workspaces of an earlier call to reuse."""
+    import paper_2607_25852_gb300 as spec
+    dev = torch.device(device)
+    d = lambda x: None if x is None else x.to(dev).contiguous()
+    S = len(bounds) - 1
+    R = B * (K + 1)
+    lg, qq = d(logits), d(q)
+    dr, sd, ri, pb, ro, dp = d(drafts), d(seeds), d(request_ids), d(pos_base), d(row_offsets), d(depth)
+    shards = []
+    for s in range(S):
+        lo, hi = bounds[s], bounds[s + 1]
+        shards.append((lo, lg[:, lo:hi].contiguous(),
+                       None if qq is None else qq[:, :, lo:hi].contiguous(),
+                       spec.shard_workspace(B, K, hi - lo, dev) if ws is None else ws[s]))
+    stats = torch.zeros(S * R * spec.SHARD_STAT_BYTES, dtype=torch.uint8, device=dev)
+    races = torch.zeros(S * B * spec.SHARD_RACE_BYTES, dtype=torch.uint8, device=dev)
+    dec = torch.zeros(B * spec.SHARD_DECISION_BYTES, dtype=torch.uint8, device=dev)
+    acc = torch.full((B,), -7, dtype=torch.int32, device=dev)
+    tok = torch.full((B, K + 1), -7, dtype=torch.int32, device=dev)
+    pdr = torch.full((B, max(K, 1)), -7.0, dtype=torch.float32, device=dev)
+    rst = torch.zeros((R, 2), dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    sb, rb = R * spec.SHARD_STAT_BYTES, B * spec.SHARD_RACE_BYTES
+    for s, (lo, lgs, qs, ws) in enumerate(shards):
+        spec.spec_shard_stats(lgs, dr, qs, B, K, V, lo, t, pb, stats[s * sb:(s + 1) * sb], ws,
+                              row_offsets=ro, depth=dp, status=status)
+    spec.spec_shard_decide(stats, S, dr, q is not None, B, K, V, t, sd, ri, pb, acc, tok,
+                           decisions_out=dec, row_offsets=ro, depth=dp,
+                           p_draft_out=pdr if K > 0 else None, row_stats_out=rst, status=status)
+    for s, (lo, lgs, qs, ws) in enumerate(shards):
+        spec.spec_shard_sample(lgs, qs, dec, B, K, V, lo, t, sd, ri, races[s * rb:(s + 1) * rb], ws,
+                               status=status)
+    spec.spec_shard_finish(races, S, dec, B, K, V, t, sd, ri, acc, tok, status=status)
+    torch.cuda.synchronize()
+    return dict(accepted=acc.cpu().numpy(), tokens=tok.cpu().numpy(), p_draft=pdr.cpu().numpy()[:, :K],
+                row_stats=rst.cpu().numpy(), status=int(status.item()),
+                ws=[w for _, _, _, w in shards])

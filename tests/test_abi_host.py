@@ -95,3 +95,34 @@ def test_argument_errors_return_before_any_launch(lib):
     assert c(2, 2, dummy, dummy, H=0) == 1
     assert c(2, 2, dummy, dummy, dt=3) == 1
     assert lib.spec_profile_stream_pass(dummy, None) == 1
+
+
+def test_shard_workspace_and_argument_errors(lib):
+    import paper_2607_25852_gb300 as spec
+    assert spec.spec_shard_workspace(0, 4, 1024) == 0
+    assert spec.spec_shard_workspace(4, 256, 1024) == 0
+    n = spec.spec_shard_workspace(64, 16, 201088 // 8)
+    assert n > 0 and n % 256 == 0 and n < (1 << 20)
+    dummy = ctypes.c_void_p(16)          # never dereferenced: every call below fails its checks
+    ws = ctypes.c_void_p(256)
+    stream = ctypes.c_void_p(0)
+    st = lambda V, vb, Vs, t=1.0, ws_bytes=1 << 20, out=dummy: lib.spec_shard_stats(
+        dummy, 0, None, None, dummy, None, 0, 4, 3, V, vb, Vs, t, dummy, out, None, ws, ws_bytes,
+        stream)
+    assert st(5000, 4096, 1024) == 1       # past V
+    assert st(5000, -1, 1024) == 1
+    assert st(5000, 0, 0) == 1
+    assert st(5000, 0, 1024, t=-1.0) == 1
+    assert st(5000, 0, 1024, ws_bytes=8) == 2
+    assert st(5000, 0, 1024, out=ctypes.c_void_p(24)) == 1   # records not 16-byte aligned
+    d = lambda S, t, dec=dummy: lib.spec_shard_decide(
+        dummy, S, None, None, dummy, 0, 4, 3, 5000, t, dummy, dummy, dummy, dummy, dummy, None, None,
+        dec, None, stream)
+    assert d(0, 1.0) == 1 and d(2, -1.0) == 1 and d(2, 1.0, dec=None) == 1
+    s = lambda vb, Vs, t: lib.spec_shard_sample(
+        dummy, 0, None, 0, dummy, 4, 3, 5000, vb, Vs, t, dummy, dummy, dummy, None, ws, 1 << 20, stream)
+    assert s(4500, 1024, 1.0) == 1
+    assert s(0, 1024, 0.0) == 0            # nothing to sample at t = 0: no launch
+    f = lambda S, t: lib.spec_shard_finish(dummy, S, dummy, 4, 3, 5000, t, dummy, dummy, dummy, dummy,
+                                           None, stream)
+    assert f(0, 1.0) == 1 and f(2, 0.0) == 0
