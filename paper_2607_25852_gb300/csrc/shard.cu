@@ -110,6 +110,7 @@ struct ShardLaunch {
   // workspace of stats / sample
   RowPartial* row_part;    // [R_max * NC]
   RacePartial* race_part;  // [B * NCS]
+  ShardPart* part_ws;      // [B][2] the cut blocks' parts (sample)
   uint32_t* row_count;     // [R_max] arrivals per row (stats)
   uint32_t* req_count;     // [B] arrivals per request (sample)
   int NC, chunk;           // stats: chunks per row and their length
@@ -121,7 +122,7 @@ struct ShardGeometry {
   int NC, chunk;  // streaming pass over V_shard columns
   int quads_s;    // race quads per sampling chunk
   int NCS_max;    // sampling chunks for any shard start
-  size_t row_part_off, race_part_off, counters_off, bytes;
+  size_t row_part_off, race_part_off, part_off, counters_off, bytes;
 };
 
 static inline size_t round256(size_t x) { return (x + 255) / 256 * 256; }
@@ -138,7 +139,8 @@ static ShardGeometry shard_geometry(int B, int K, int Vs) {
   const size_t R_max = (size_t)B * (K + 1);
   s.row_part_off = 0;
   s.race_part_off = round256(sizeof(RowPartial) * R_max * s.NC);
-  s.counters_off = s.race_part_off + round256(sizeof(RacePartial) * (size_t)B * s.NCS_max);
+  s.part_off = s.race_part_off + round256(sizeof(RacePartial) * (size_t)B * s.NCS_max);
+  s.counters_off = s.part_off + round256(sizeof(ShardPart) * 2 * (size_t)B);
   s.bytes = s.counters_off + round256(sizeof(uint32_t) * (R_max + (size_t)B));
   return s;
 }
@@ -147,6 +149,40 @@ static ShardGeometry shard_geometry(int B, int K, int Vs) {
 // spec_shard_stats: one CTA per (request, row, chunk of the shard); the last
 // CTA of a row to finish merges the row's chunk partials into its record.
 // ---------------------------------------------------------------------------
+// The row's draft, seen from this shard: its logit and q value if the shard
+// owns the draft's column.  Loaded before the stream, used after it.
+struct DraftView {
+  float lz, qz;
+  int32_t owned;
+};
+template <typename T>
+__device__ __forceinline__ DraftView draft_view(const ShardLaunch& p, int i, int j, const ReqShape& rs, const T* row) {
+  DraftView d{0.0f, 1.0f, 0};
+  if (j < rs.n) {
+    const int z = __ldg(p.drafts + (size_t)i * p.K + j);
+    if (z >= p.v_begin && z < p.v_begin + p.Vs) {
+      d.owned = 1;
+      d.lz = load_elem(row + (z - p.v_begin));
+      if (p.dense_q) d.qz = load_any(p.q, p.q_dtype, ((int64_t)i * p.K + j) * (int64_t)p.Vs + (z - p.v_begin));
+    }
+  }
+  return d;
+}
+
+__device__ __forceinline__ void write_stat(const ShardLaunch& p, long long r, float m, float s, int32_t idx,
+                                           int32_t flags, const DraftView& d) {
+  ShardStat st;
+  st.m = m;
+  st.s = s;
+  st.idx = idx;
+  st.flags = flags;
+  st.lz = d.lz;
+  st.qz = d.qz;
+  st.owned = d.owned;
+  st.pad = 0;
+  p.stats[r] = st;
+}
+
 template <typename T, bool kGreedy>
 __global__ void __launch_bounds__(kStreamThreads) shard_stats_kernel(const ShardLaunch p) {
   const int per_req = (p.K + 1) * p.NC;
@@ -160,10 +196,16 @@ __global__ void __launch_bounds__(kStreamThreads) shard_stats_kernel(const Shard
   pdl_launch_dependents();
   const long long r = rs.row0 + j;
   const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.Vs;
+  DraftView dv{0.0f, 1.0f, 0};
+  if (threadIdx.x == 0) dv = draft_view(p, i, j, rs, row);
   RowAcc<T, kGreedy> acc;
   const int v0 = c * p.chunk;
   stream_chunk<T, kGreedy>(acc, row, v0, min(p.Vs, v0 + p.chunk), p.v_begin, p.c2);
   const RowPartial part = cta_reduce_partial<T, kGreedy>(acc, p.c2);
+  if (p.NC == 1) {  // the whole shard row in this CTA: its partial is the record
+    if (threadIdx.x == 0) write_stat(p, r, part.m, part.s, kGreedy ? part.idx : INT_MAX, part.flags, dv);
+    return;
+  }
   __shared__ int sh_last;
   if (threadIdx.x == 0) {
     p.row_part[(size_t)r * p.NC + c] = part;
@@ -211,18 +253,7 @@ __global__ void __launch_bounds__(kStreamThreads) shard_stats_kernel(const Shard
   }
   st.flags = (int32_t)__reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
   if (lane == 0) {
-    st.lz = 0.0f;
-    st.qz = 1.0f;
-    st.owned = 0;
-    if (j < rs.n) {
-      const int z = __ldg(p.drafts + (size_t)i * p.K + j);
-      if (z >= p.v_begin && z < p.v_begin + p.Vs) {
-        st.owned = 1;
-        st.lz = load_elem(row + (z - p.v_begin));
-        if (p.dense_q) st.qz = load_any(p.q, p.q_dtype, ((int64_t)i * p.K + j) * (int64_t)p.Vs + (z - p.v_begin));
-      }
-    }
-    p.stats[r] = st;
+    write_stat(p, r, st.m, st.s, st.idx, st.flags, dv);
     p.row_count[r] = 0u;  // leave the workspace zeroed for the next call
   }
 }
@@ -240,6 +271,7 @@ __global__ void __launch_bounds__(32) shard_decide_kernel(const ShardLaunch p) {
   __shared__ int32_t sh_g[kMaxRows];
   __shared__ int32_t sh_z[kMaxRows];
   __shared__ float sh_pz[kMaxRows];
+  __shared__ float sh_lq[kMaxRows];
   const ReqShape rs = request_shape(p, i);
   const DecidePre pre = decide_prefetch(p, i);
   const int n = rs.n;
@@ -256,48 +288,67 @@ __global__ void __launch_bounds__(32) shard_decide_kernel(const ShardLaunch p) {
     qz[u] = 1.0f;
   }
   if (rs.valid) {
-    // rows (a lane per row): the S shard records merged in shard order
+    // rows (a lane per row): the S shard records merged in shard order, their
+    // loads issued kBatch at a time; the draft fields come with them
+    constexpr int kBatch = 8;
+    const uint4* rec = reinterpret_cast<const uint4*>(p.stats);
     for (int j = lane; j <= n; j += 32) {
       int32_t f = 0;
-      if (kGreedy) {
-        ArgState best{-INFINITY, INT_MAX};
-        for (int s = 0; s < p.S; ++s) {
-          const ShardStat st = p.stats[(size_t)s * p.R_max + row0 + j];
-          f |= st.flags;
-          ArgState o{st.m, st.idx};
-          if (arg_better(o, best)) best = o;
+      ArgState best{-INFINITY, INT_MAX};
+      SoftState all{-INFINITY, 0.0f};
+      int owners = 0;
+      float lzj = 0.0f, qzj = 1.0f;
+      for (int s0 = 0; s0 < p.S; s0 += kBatch) {
+        uint4 a[kBatch], b[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          if (s0 + u < p.S) {
+            const size_t k = 2 * ((size_t)(s0 + u) * p.R_max + row0 + j);
+            a[u] = rec[k];
+            if (j < n) b[u] = rec[k + 1];
+          }
         }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          if (s0 + u >= p.S) break;
+          f |= (int32_t)a[u].w;
+          if (kGreedy) {
+            const ArgState o{__uint_as_float(a[u].x), (int32_t)a[u].z};
+            if (arg_better(o, best)) best = o;
+          } else {
+            all = soft_merge(all, SoftState{__uint_as_float(a[u].x), __uint_as_float(a[u].y)}, p.c2);
+          }
+          if (j < n && b[u].z) {
+            ++owners;
+            lzj = __uint_as_float(b[u].x);
+            qzj = __uint_as_float(b[u].y);
+          }
+        }
+      }
+      if (kGreedy) {
         sh_m[j] = best.v;
         sh_g[j] = best.idx;
         if (f || best.idx == INT_MAX) bad = 1;
       } else {
-        SoftState all{-INFINITY, 0.0f};
-        for (int s = 0; s < p.S; ++s) {
-          const ShardStat st = p.stats[(size_t)s * p.R_max + row0 + j];
-          f |= st.flags;
-          all = soft_merge(all, SoftState{st.m, st.s}, p.c2);
-        }
         sh_m[j] = all.m;
         sh_S[j] = all.s;
+        sh_pz[j] = lzj;  // staged here; decide_chain overwrites it with p(z)
+        sh_lq[j] = qzj;
         if (f || !(all.m > -INFINITY) || !(all.s > 0.0f) || !isfinite(all.s)) bad = 1;
       }
+      // the shards must cover the draft's column exactly once
+      if (j < n && (owners != 1 || sh_z[j] < 0 || sh_z[j] >= p.V)) bad = 1;
     }
-    // drafts (a lane per draft): the owning shard's logit and q value
+    if (!kGreedy) {
+      __syncwarp();
 #pragma unroll
-    for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
-      const int j = lane + 32 * u;
-      if (j >= n) break;
-      int owners = 0;
-      for (int s = 0; s < p.S; ++s) {
-        const ShardStat st = p.stats[(size_t)s * p.R_max + row0 + j];
-        if (st.owned) {
-          ++owners;
-          lz[u] = st.lz;
-          qz[u] = st.qz;
+      for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
+        const int j = lane + 32 * u;
+        if (j < n) {
+          lz[u] = sh_pz[j];
+          qz[u] = sh_lq[j];
         }
       }
-      const int z = sh_z[j];
-      if (owners != 1 || z < 0 || z >= p.V) bad = 1;  // the shards must cover the vocabulary once
     }
   }
   bad = __any_sync(0xFFFFFFFFu, bad);
@@ -393,6 +444,22 @@ __device__ ShardPart shard_part(const ShardLaunch& p, int mode, const T* row, co
   return out;
 }
 
+// A part written by another CTA of this grid: read at L2 (.cg).
+__device__ __forceinline__ ShardPart load_part_cg(const ShardPart* ptr) {
+  const uint4 a = __ldcg(reinterpret_cast<const uint4*>(ptr));
+  const uint4 b = __ldcg(reinterpret_cast<const uint4*>(ptr) + 1);
+  ShardPart x;
+  x.blk = (int32_t)a.x;
+  x.w_r = __uint_as_float(a.y);
+  x.w_p = __uint_as_float(a.z);
+  x.ek_r = __uint_as_float(a.w);
+  x.ey_r = (int32_t)b.x;
+  x.ek_p = __uint_as_float(b.y);
+  x.ey_p = (int32_t)b.z;
+  x.pad = (int32_t)b.w;
+  return x;
+}
+
 __device__ __forceinline__ ShardPart no_part() {
   ShardPart n;
   n.blk = INT_MAX;
@@ -449,6 +516,21 @@ __global__ void __launch_bounds__(kSampleThreads, 4) shard_sample_kernel(const S
     shard_level1<T, kWeightP, false>(p, row, qrow, q_first, q_end, ra, best, best_p);
   best = cta_min_key(best, sh_red);
   if (mode != kWeightP) best_p = cta_min_key(best_p, sh_red);
+  // ---- the cut blocks at the shard's ends: the first and the last chunk's
+  // CTA compute the shard's part of each before arriving ----
+  const int hb = p.v_begin / kRaceBlock;   // block holding the first column
+  const int tb = (vend - 1) / kRaceBlock;  // block holding the last column
+  const bool head_part = p.v_begin % kRaceBlock != 0 || (vend < p.V && vend % kRaceBlock != 0 && tb == hb);
+  const bool tail_part = vend < p.V && vend % kRaceBlock != 0 && tb != hb;
+  if (cs == 0 && head_part) {
+    const ShardPart pt = shard_part<T>(p, mode, row, qrow, hb, p.v_begin, tb == hb ? vend : (hb + 1) * kRaceBlock,
+                                       ra, sh_red, sh_f);
+    if (threadIdx.x == 0) p.part_ws[2 * (size_t)i] = pt;
+  }
+  if (cs == p.NCS - 1 && tail_part) {
+    const ShardPart pt = shard_part<T>(p, mode, row, qrow, tb, tb * kRaceBlock, vend, ra, sh_red, sh_f);
+    if (threadIdx.x == 0) p.part_ws[2 * (size_t)i + 1] = pt;
+  }
   if (threadIdx.x == 0) {
     RacePartial rp;
     rp.key_r = best.key;
@@ -489,16 +571,9 @@ __global__ void __launch_bounds__(kSampleThreads, 4) shard_sample_kernel(const S
   }
   __syncthreads();
   const int b = sh_b, bp = sh_bp;
-  // ---- the straddling blocks at the shard's ends ----
   ShardPart part[2] = {no_part(), no_part()};
-  const int hb = p.v_begin / kRaceBlock;   // block holding the first column
-  const int tb = (vend - 1) / kRaceBlock;  // block holding the last column
-  const bool head_cut = p.v_begin % kRaceBlock != 0;
-  const bool tail_cut = vend < p.V && vend % kRaceBlock != 0;
-  if (head_cut || (tail_cut && tb == hb))
-    part[0] = shard_part<T>(p, mode, row, qrow, hb, p.v_begin, tb == hb ? vend : (hb + 1) * kRaceBlock, ra, sh_red,
-                            sh_f);
-  if (tail_cut && tb != hb) part[1] = shard_part<T>(p, mode, row, qrow, tb, tb * kRaceBlock, vend, ra, sh_red, sh_f);
+  if (head_part) part[0] = load_part_cg(p.part_ws + 2 * (size_t)i);
+  if (tail_part) part[1] = load_part_cg(p.part_ws + 2 * (size_t)i + 1);
   const bool empty = b == INT_MAX && !(part[0].w_r > 0.0f) && !(part[1].w_r > 0.0f);
   // ---- level 2 in the best whole block ----
   ShardRace out;
@@ -527,7 +602,7 @@ __global__ void __launch_bounds__(kSampleThreads, 4) shard_sample_kernel(const S
 }
 
 // ---------------------------------------------------------------------------
-// spec_shard_finish: one thread per request.
+// spec_shard_finish: one warp per request.
 // ---------------------------------------------------------------------------
 // Candidate block b with weight sum W (summed over its parts): key E_b / W.
 __device__ __forceinline__ void finish_block(KeyState& best, int& y, int b, float W, int y_part, const RaceArgs& a) {
@@ -541,14 +616,20 @@ __device__ __forceinline__ void finish_block(KeyState& best, int& y, int b, floa
   }
 }
 
-__global__ void __launch_bounds__(128) shard_finish_kernel(const ShardLaunch p) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+// One warp per request: the lanes load up to 32 shards' records at a time
+// into shared memory, lane 0 merges them in shard order.
+constexpr int kFinishWarps = 4;
+
+__global__ void __launch_bounds__(32 * kFinishWarps) shard_finish_kernel(const ShardLaunch p) {
+  __shared__ ShardRace sh_rec[kFinishWarps][32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * kFinishWarps + warp;
   pdl_wait_prerequisites();
   if (i >= p.B) return;
   const ReqRec rec = p.req_rec[i];
   if (rec.flags & 1) return;
   if (rec.a < 0 || rec.a > p.K) {
-    report(p.status, SPEC_ERR_WORKSPACE);
+    if (lane == 0) report(p.status, SPEC_ERR_WORKSPACE);
     return;
   }
   RaceArgs a{};
@@ -559,40 +640,52 @@ __global__ void __launch_bounds__(128) shard_finish_kernel(const ShardLaunch p) 
   a.k1 = (uint32_t)(seed >> 32);
   KeyState r{INFINITY, INT_MAX}, q{INFINITY, INT_MAX};
   int yr = -1, yq = -1;
-  // straddling blocks: the parts of one block are adjacent in shard order
+  // cut blocks: the parts of one block are adjacent in shard order
   int cur = INT_MAX;
   float Wr = 0.0f, Wp = 0.0f;
   KeyState er{INFINITY, INT_MAX}, ep{INFINITY, INT_MAX};
-  for (int s = 0; s < p.S; ++s) {
-    const ShardRace& x = p.races[(size_t)s * p.B + i];
-    const KeyState kr{x.key_r, x.blk_r}, kp{x.key_p, x.blk_p};
-    if (x.blk_r != INT_MAX && key_better(kr, r)) {
-      r = kr;
-      yr = x.y_r;
+  for (int s0 = 0; s0 < p.S; s0 += 32) {
+    __syncwarp();
+    if (s0 + lane < p.S) {
+      const uint4* src = reinterpret_cast<const uint4*>(p.races + (size_t)(s0 + lane) * p.B + i);
+      uint4* dst = reinterpret_cast<uint4*>(&sh_rec[warp][lane]);
+#pragma unroll
+      for (int w = 0; w < (int)(sizeof(ShardRace) / 16); ++w) dst[w] = src[w];
     }
-    if (x.blk_p != INT_MAX && key_better(kp, q)) {
-      q = kp;
-      yq = x.y_p;
-    }
-    for (int h = 0; h < 2; ++h) {
-      const ShardPart& pt = x.part[h];
-      if (pt.blk == INT_MAX) continue;
-      if (pt.blk != cur) {
-        if (cur != INT_MAX) {
-          finish_block(r, yr, cur, Wr, er.idx, a);
-          finish_block(q, yq, cur, Wp, ep.idx, a);
-        }
-        cur = pt.blk;
-        Wr = Wp = 0.0f;
-        er = ep = KeyState{INFINITY, INT_MAX};
+    __syncwarp();
+    if (lane != 0) continue;
+    for (int s = s0; s < min(p.S, s0 + 32); ++s) {
+      const ShardRace& x = sh_rec[warp][s - s0];
+      const KeyState kr{x.key_r, x.blk_r}, kp{x.key_p, x.blk_p};
+      if (x.blk_r != INT_MAX && key_better(kr, r)) {
+        r = kr;
+        yr = x.y_r;
       }
-      Wr += pt.w_r;
-      Wp += pt.w_p;
-      const KeyState kr2{pt.ek_r, pt.ey_r}, kp2{pt.ek_p, pt.ey_p};
-      if (pt.ey_r != INT_MAX && key_better(kr2, er)) er = kr2;
-      if (pt.ey_p != INT_MAX && key_better(kp2, ep)) ep = kp2;
+      if (x.blk_p != INT_MAX && key_better(kp, q)) {
+        q = kp;
+        yq = x.y_p;
+      }
+      for (int h = 0; h < 2; ++h) {
+        const ShardPart& pt = x.part[h];
+        if (pt.blk == INT_MAX) continue;
+        if (pt.blk != cur) {
+          if (cur != INT_MAX) {
+            finish_block(r, yr, cur, Wr, er.idx, a);
+            finish_block(q, yq, cur, Wp, ep.idx, a);
+          }
+          cur = pt.blk;
+          Wr = Wp = 0.0f;
+          er = ep = KeyState{INFINITY, INT_MAX};
+        }
+        Wr += pt.w_r;
+        Wp += pt.w_p;
+        const KeyState kr2{pt.ek_r, pt.ey_r}, kp2{pt.ek_p, pt.ey_p};
+        if (pt.ey_r != INT_MAX && key_better(kr2, er)) er = kr2;
+        if (pt.ey_p != INT_MAX && key_better(kp2, ep)) ep = kp2;
+      }
     }
   }
+  if (lane != 0) return;
   if (cur != INT_MAX) {
     finish_block(r, yr, cur, Wr, er.idx, a);
     finish_block(q, yq, cur, Wp, ep.idx, a);
@@ -755,6 +848,7 @@ extern "C" int spec_shard_sample(const void* logits_shard, int logits_dtype, con
   p.status = status;
   char* base = static_cast<char*>(ws);
   p.race_part = reinterpret_cast<spec::RacePartial*>(base + g.race_part_off);
+  p.part_ws = reinterpret_cast<spec::ShardPart*>(base + g.part_off);
   p.req_count = reinterpret_cast<uint32_t*>(base + g.counters_off) + (size_t)B * (K + 1);
   // the shard's quads, in chunks of quads_s
   p.q0 = v_begin / spec::kRaceQuad;
@@ -799,7 +893,8 @@ extern "C" int spec_shard_finish(const void* races, int S, const void* decisions
   p.out_tokens = out_tokens;
   p.status = status;
   const cudaError_t err =
-      spec::launch_after_previous(spec::shard_finish_kernel, dim3((B + 127) / 128), dim3(128), 0, stream, p);
+      spec::launch_after_previous(spec::shard_finish_kernel, dim3((B + spec::kFinishWarps - 1) / spec::kFinishWarps),
+                                  dim3(32 * spec::kFinishWarps), 0, stream, p);
   if (err != cudaSuccess || cudaGetLastError() != cudaSuccess) return SPEC_ERR_CUDA;
   return SPEC_OK;
 }
