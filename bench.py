@@ -56,6 +56,8 @@ def parse():
     ap.add_argument("--no-graph", action="store_true", help="skip the CUDA-graph replay timing")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--shards", type=int, default=1,
+                    help="S > 1: time vocabulary-sharded verification with S shards emulated on one GPU")
     return ap.parse_args()
 
 
@@ -530,10 +532,111 @@ def run_ours(args):
     return 0
 
 
+def run_sharded(args):
+    """Vocabulary-sharded verification (the target's TP layout) with the S
+    shards on this one GPU: the whole round (S x stats, decide, S x sample,
+    finish; the records written side by side in place of the all-gathers),
+    and the per-rank critical path (shard 0's stats and sample, decide,
+    finish), each call timed alone."""
+    import torch
+    import paper_2607_25852_gb300 as spec
+    from paper_2607_25852_gb300.sharded import ShardedRound, even_bounds
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    wl = make_inputs(args, 0, device)
+    B, K, V, t = wl.B, wl.K, wl.V, wl.temperature
+    S = args.shards
+    bounds = even_bounds(V, S)
+    rnd = ShardedRound(B, K, V, bounds, device=device, local=True)
+    lgs = [wl.logits[:, bounds[s]:bounds[s + 1]].contiguous() for s in range(S)]
+    qs = None if wl.q is None else [wl.q[:, :, bounds[s]:bounds[s + 1]].contiguous() for s in range(S)]
+    acc = torch.zeros(B, dtype=torch.int32, device=device)
+    tok = torch.zeros((B, K + 1), dtype=torch.int32, device=device)
+    status = torch.zeros(1, dtype=torch.int32, device=device)
+    stream = torch.cuda.current_stream()
+
+    def round_():
+        rnd.run(lgs, wl.drafts, qs, t, wl.seeds, wl.request_ids, wl.pos_base, acc, tok, status=status)
+
+    for _ in range(max(args.warmup, 3)):
+        round_()
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, "device reported an input error"
+    R = B * (K + 1)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clocks:
+        a.record(stream)
+        for _ in range(args.steps):
+            round_()
+        b.record(stream)
+        torch.cuda.synchronize()
+    round_ms = a.elapsed_time(b) / args.steps
+
+    # per-rank calls of shard 0, each bracketed by its own events
+    sb, rb = R * spec.SHARD_STAT_BYTES, B * spec.SHARD_RACE_BYTES
+    q0 = None if qs is None else qs[0]
+    calls = {
+        "stats": lambda: spec.spec_shard_stats(lgs[0], wl.drafts, q0, B, K, V, 0, t, wl.pos_base,
+                                               rnd.stats[:sb], rnd.ws[0], status=status),
+        "decide": lambda: spec.spec_shard_decide(rnd.stats, S, wl.drafts, q0 is not None, B, K, V, t, wl.seeds,
+                                                 wl.request_ids, wl.pos_base, acc, tok,
+                                                 decisions_out=rnd.decisions, status=status),
+        "sample": lambda: spec.spec_shard_sample(lgs[0], q0, rnd.decisions, B, K, V, 0, t, wl.seeds,
+                                                 wl.request_ids, rnd.races[:rb], rnd.ws[0], status=status),
+        "finish": lambda: spec.spec_shard_finish(rnd.races, S, rnd.decisions, B, K, V, t, wl.seeds,
+                                                 wl.request_ids, acc, tok, status=status),
+    }
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=device)
+    per = {}
+    for name, fn in calls.items():
+        if t == 0 and name in ("sample", "finish"):
+            continue
+        ts = []
+        for k in range(args.steps):
+            round_()                    # leaves every record of this round in place
+            flush.fill_(k & 0xFF)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        per[name] = 1e3 * statistics.median(ts)
+    assert int(status.item()) == 0
+    peak, peak_kind = measured_peak()
+    esize = 2 if wl.dtype == "bf16" else 4
+    stats_bytes = R * (bounds[1] - bounds[0]) * esize
+    achieved = stats_bytes / (per["stats"] * 1e-6) / 1e9
+    line = {
+        "metric": METRIC, "value": R * args.steps / (round_ms * 1e-3 * args.steps), "unit": UNIT,
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
+        "data": "synthetic",
+        "config": {"workload": f"{wl.name}: B={B} K={K} V={V} {wl.dtype} logits, t={t}, "
+                               f"q {'bf16 [B,K,V]' if wl.q is not None else 'one-hot'}",
+                   "shards": S, "bounds": bounds,
+                   "parallelism": f"vocabulary split into {S} shards, all on one GPU (records written "
+                                  "side by side in place of the all-gathers)"},
+        "per_rank_us": {k: round(v, 2) for k, v in per.items()},
+        "per_rank_critical_path_us": round(sum(per.values()), 2),
+        "exchange_bytes_per_rank": {"stats": sb, "races": rb if t > 0 else 0},
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": None, "kernel": "shard_stats_kernel",
+                     "peak_kind": peak_kind, "algorithmic_bytes_per_launch": stats_bytes,
+                     "avg_launch_us": round(per["stats"], 2)},
+        "clocks": clocks.summary(),
+        "gpu_launches": (2 * S + 2 if t > 0 else S + 1) * args.steps,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.shards > 1:
+        return run_sharded(args)
     return run_ours(args)
 
 

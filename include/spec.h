@@ -14,6 +14,8 @@
  *   spec_commit    packing of the committed tokens and of the target hidden
  *                  rows that condition the drafter's next round (Sections 1,
  *                  3.1 and 6).
+ *   spec_shard_*   spec_verify for a target whose vocabulary is split over
+ *                  tensor-parallel ranks (Section 4.4 serves with TP = 8).
  *
  * Conventions shared by every entry point
  *   - Pointers marked "device" are CUDA device (or managed) memory of the

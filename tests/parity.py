@@ -124,42 +124,27 @@ def shard_bounds(V, S, unit=1):
 
 def run_sharded(logits, drafts, q, B, K, V, t, seeds, request_ids, pos_base, bounds,
                 row_offsets=None, depth=None, ws=None, device="cuda"):
-    """The four shard calls over shards [bounds[s], bounds[s+1]) of one GPU;
-    the records of the S shards are written side by side (the exchange).
-    `ws`: the per-shard workspaces of an earlier call to reuse."""
-    import paper_2607_25852_gb300 as spec
+    """The four shard calls over shards [bounds[s], bounds[s+1]) of one GPU
+    (paper_2607_25852_gb300.sharded.ShardedRound with local=True: the S
+    shards' records are written side by side, in place of the exchanges).
+    `ws`: the ShardedRound of an earlier call, to reuse its workspaces."""
+    from paper_2607_25852_gb300.sharded import ShardedRound
     dev = torch.device(device)
     d = lambda x: None if x is None else x.to(dev).contiguous()
     S = len(bounds) - 1
     R = B * (K + 1)
     lg, qq = d(logits), d(q)
-    dr, sd, ri, pb, ro, dp = d(drafts), d(seeds), d(request_ids), d(pos_base), d(row_offsets), d(depth)
-    shards = []
-    for s in range(S):
-        lo, hi = bounds[s], bounds[s + 1]
-        shards.append((lo, lg[:, lo:hi].contiguous(),
-                       None if qq is None else qq[:, :, lo:hi].contiguous(),
-                       spec.shard_workspace(B, K, hi - lo, dev) if ws is None else ws[s]))
-    stats = torch.zeros(S * R * spec.SHARD_STAT_BYTES, dtype=torch.uint8, device=dev)
-    races = torch.zeros(S * B * spec.SHARD_RACE_BYTES, dtype=torch.uint8, device=dev)
-    dec = torch.zeros(B * spec.SHARD_DECISION_BYTES, dtype=torch.uint8, device=dev)
+    rnd = ShardedRound(B, K, V, bounds, device=dev, local=True) if ws is None else ws
+    lgs = [lg[:, bounds[s]:bounds[s + 1]].contiguous() for s in range(S)]
+    qs = None if qq is None else [qq[:, :, bounds[s]:bounds[s + 1]].contiguous() for s in range(S)]
     acc = torch.full((B,), -7, dtype=torch.int32, device=dev)
     tok = torch.full((B, K + 1), -7, dtype=torch.int32, device=dev)
     pdr = torch.full((B, max(K, 1)), -7.0, dtype=torch.float32, device=dev)
     rst = torch.zeros((R, 2), dtype=torch.float32, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    sb, rb = R * spec.SHARD_STAT_BYTES, B * spec.SHARD_RACE_BYTES
-    for s, (lo, lgs, qs, ws) in enumerate(shards):
-        spec.spec_shard_stats(lgs, dr, qs, B, K, V, lo, t, pb, stats[s * sb:(s + 1) * sb], ws,
-                              row_offsets=ro, depth=dp, status=status)
-    spec.spec_shard_decide(stats, S, dr, q is not None, B, K, V, t, sd, ri, pb, acc, tok,
-                           decisions_out=dec, row_offsets=ro, depth=dp,
-                           p_draft_out=pdr if K > 0 else None, row_stats_out=rst, status=status)
-    for s, (lo, lgs, qs, ws) in enumerate(shards):
-        spec.spec_shard_sample(lgs, qs, dec, B, K, V, lo, t, sd, ri, races[s * rb:(s + 1) * rb], ws,
-                               status=status)
-    spec.spec_shard_finish(races, S, dec, B, K, V, t, sd, ri, acc, tok, status=status)
+    rnd.run(lgs, d(drafts), qs, t, d(seeds), d(request_ids), d(pos_base), acc, tok,
+            row_offsets=d(row_offsets), depth=d(depth), p_draft_out=pdr if K > 0 else None,
+            row_stats_out=rst, status=status)
     torch.cuda.synchronize()
     return dict(accepted=acc.cpu().numpy(), tokens=tok.cpu().numpy(), p_draft=pdr.cpu().numpy()[:, :K],
-                row_stats=rst.cpu().numpy(), status=int(status.item()),
-                ws=[w for _, _, _, w in shards])
+                row_stats=rst.cpu().numpy(), status=int(status.item()), ws=rnd)

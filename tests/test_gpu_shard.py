@@ -147,14 +147,38 @@ def test_bad_inputs_are_flagged_per_request():
 
 
 def test_uncovered_draft_column_is_flagged():
-    """Shards that leave a draft's column uncovered: the request is flagged."""
+    """Shards that leave a draft's column uncovered (called through the C ABI
+    directly: ShardedRound refuses such bounds): the request is flagged."""
     import paper_2607_25852_gb300 as spec
     wl = _random_case(2048, "f32", 1.0, "onehot", B=3, K=2, seed=27)
     wl.drafts[1, 0] = 2047
-    gpu = run_sharded(wl.logits, wl.drafts, None, wl.B, wl.K, wl.V, 1.0, wl.seeds, wl.request_ids,
-                      wl.pos_base, [0, 1024, 2047])
-    assert gpu["status"] == spec.ERR_BAD_INPUT
-    assert gpu["accepted"][1] == 0 and (gpu["tokens"][1] == -1).all()
+    B, K, V = wl.B, wl.K, wl.V
+    dev = torch.device("cuda")
+    d = lambda x: x.to(dev).contiguous()
+    bounds = [0, 1024, 2047]
+    R = B * (K + 1)
+    stats = torch.zeros(2 * R * spec.SHARD_STAT_BYTES, dtype=torch.uint8, device=dev)
+    races = torch.zeros(2 * B * spec.SHARD_RACE_BYTES, dtype=torch.uint8, device=dev)
+    dec = torch.zeros(B * spec.SHARD_DECISION_BYTES, dtype=torch.uint8, device=dev)
+    acc = torch.zeros(B, dtype=torch.int32, device=dev)
+    tok = torch.zeros((B, K + 1), dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    dr, sd, ri, pb = d(wl.drafts), d(wl.seeds), d(wl.request_ids), d(wl.pos_base)
+    lgs = [d(wl.logits[:, bounds[s]:bounds[s + 1]]) for s in range(2)]
+    ws = [spec.shard_workspace(B, K, bounds[s + 1] - bounds[s], dev) for s in range(2)]
+    sb, rb = R * spec.SHARD_STAT_BYTES, B * spec.SHARD_RACE_BYTES
+    for s in range(2):
+        spec.spec_shard_stats(lgs[s], dr, None, B, K, V, bounds[s], 1.0, pb, stats[s * sb:(s + 1) * sb], ws[s],
+                              status=status)
+    spec.spec_shard_decide(stats, 2, dr, False, B, K, V, 1.0, sd, ri, pb, acc, tok, decisions_out=dec,
+                           status=status)
+    for s in range(2):
+        spec.spec_shard_sample(lgs[s], None, dec, B, K, V, bounds[s], 1.0, sd, ri, races[s * rb:(s + 1) * rb],
+                               ws[s], status=status)
+    spec.spec_shard_finish(races, 2, dec, B, K, V, 1.0, sd, ri, acc, tok, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == spec.ERR_BAD_INPUT
+    assert int(acc[1]) == 0 and (tok[1] == -1).all()
 
 
 def test_full_size_tp8_stress():
