@@ -63,6 +63,9 @@ def _declare(lib):
         ctypes.c_int, ctypes.c_double, _P, _P, _P,
         _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.oracle_verify_batch.restype = ctypes.c_int
+    lib.oracle_draft_batch.argtypes = [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                       ctypes.c_double, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
+    lib.oracle_draft_batch.restype = ctypes.c_int
     lib.oracle_budget.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, ctypes.c_int64]
     lib.oracle_budget.restype = ctypes.c_int
     lib.oracle_allocate.argtypes = [
@@ -218,6 +221,28 @@ def verify_batch(logits, drafts, q, t, seeds, request_ids, pos_base,
         out["race"][i] = res["race"]
         out["mode"][i] = res["mode"]
         out["status"][i] = res["status"]
+    return out
+
+
+# --------------------------------------------------------------------------
+# The drafter's producer step
+# --------------------------------------------------------------------------
+def draft_batch(logits, tau, seeds, request_ids, pos_base):
+    """Drafts, confidences and D-cut scores from the drafter's logits
+    [B, K, V] (see oracle_draft_request in spec_oracle.c)."""
+    logits = _c(logits)
+    B, K, V = logits.shape
+    seeds = _c(seeds, np.uint64)
+    request_ids = _c(request_ids, np.uint64)
+    pos_base = _c(pos_base, np.int64)
+    out = dict(z=np.full((B, K), -1, np.int32), c=np.zeros((B, K), np.float64),
+               s=np.zeros((B, K + 1), np.float32), m=np.zeros((B, K), np.float64),
+               logS=np.zeros((B, K), np.float64), race=np.zeros((B, K, 9), np.float64),
+               status=np.zeros(B, np.int32))
+    load().oracle_draft_batch(
+        _ptr(logits), _dtype_code(logits), B, K, V, float(tau), _ptr(seeds), _ptr(request_ids),
+        _ptr(pos_base), _ptr(out["z"]), _ptr(out["c"]), _ptr(out["s"]), _ptr(out["m"]),
+        _ptr(out["logS"]), _ptr(out["race"]), _ptr(out["status"]))
     return out
 
 

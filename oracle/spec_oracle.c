@@ -45,7 +45,8 @@
  *   counter = (lo32(position), lo32(request), hi32(request), purpose<<28 | sub)
  *   purpose ACCEPT = 1 (sub = 0, word 0 used), SAMPLE = 2 (block variates:
  *   sub = b / 4, word b % 4), SAMPLE_IN_BLOCK = 3 (entry variates: sub = v / 4,
- *   word v % 4).  Acceptance uniform: (x >> 8) * 2^-24.  Race variate:
+ *   word v % 4); the drafter's draw uses DRAFT = 4 and DRAFT_IN_BLOCK = 5 in
+ *   the same way.  Acceptance uniform: (x >> 8) * 2^-24.  Race variate:
  *   E = -ln((2 * (x >> 9) + 1) * 2^-24), the midpoint of one of 2^23 equal
  *   cells of (0, 1), so that E > 0: a variate of exactly 0 would make its entry
  *   win whatever its weight, and the draw would no longer follow w / sum(w).
@@ -73,6 +74,8 @@
 #define OR_PURPOSE_ACCEPT 1u
 #define OR_PURPOSE_SAMPLE 2u
 #define OR_PURPOSE_SAMPLE_IN_BLOCK 3u
+#define OR_PURPOSE_DRAFT 4u          /* the drafter's draw: block variates */
+#define OR_PURPOSE_DRAFT_IN_BLOCK 5u /* the drafter's draw: entry variates */
 #define OR_RACE_BLOCK 256
 
 /* ------------------------------------------------------------------------ */
@@ -147,25 +150,34 @@ double oracle_race_variate(uint32_t word) {
   return -log(u);
 }
 
+/* Exponential variate number `index` of purpose `purpose` at `position`:
+ * word index % 4 of the Philox call with sub-index index / 4. */
+static double race_exponential_with(uint64_t seed, uint64_t request,
+                                    uint64_t position, uint32_t purpose,
+                                    uint32_t index) {
+  uint32_t w[4];
+  draw_words(seed, request, position, purpose, index >> 2, w);
+  return oracle_race_variate(w[index & 3u]);
+}
+
 /* Exponential variate of the sampling race at `position`: level 1 (block b,
  * level = 1) or level 2 (entry v, level = 2). */
 double oracle_race_exponential(uint64_t seed, uint64_t request,
                                uint64_t position, uint32_t index, int level) {
-  uint32_t w[4];
-  draw_words(seed, request, position,
-             level == 1 ? OR_PURPOSE_SAMPLE : OR_PURPOSE_SAMPLE_IN_BLOCK,
-             index >> 2, w);
-  return oracle_race_variate(w[index & 3u]);
+  return race_exponential_with(seed, request, position,
+                               level == 1 ? OR_PURPOSE_SAMPLE : OR_PURPOSE_SAMPLE_IN_BLOCK,
+                               index);
 }
 
-/* Two-level exponential race over weights w[0..V) (see the file header).
+/* Two-level exponential race over weights w[0..V) (see the file header),
+ * with block variates of purpose `pb` and entry variates of purpose `pe`.
  * race_out[9]: best block key, best block, second block key, second block,
  * the winner y in the best block, its key, the second key in that block, the
  * second entry in that block, and the winner in the second block (-1 if
  * none).  Returns y, or -1 if every weight is zero. */
-static int two_level_race(const double* w, int V, uint64_t seed,
-                          uint64_t request, uint64_t position,
-                          double* race_out) {
+static int two_level_race_with(const double* w, int V, uint64_t seed,
+                               uint64_t request, uint64_t position,
+                               uint32_t pb, uint32_t pe, double* race_out) {
   const int nb = (V + OR_RACE_BLOCK - 1) / OR_RACE_BLOCK;
   double b1k = INFINITY, b2k = INFINITY;
   int b1 = -1, b2 = -1;
@@ -174,7 +186,7 @@ static int two_level_race(const double* w, int V, uint64_t seed,
     for (int v = b * OR_RACE_BLOCK; v < V && v < (b + 1) * OR_RACE_BLOCK; ++v)
       W += w[v];
     if (!(W > 0.0)) continue;
-    double key = oracle_race_exponential(seed, request, position, (uint32_t)b, 1) / W;
+    double key = race_exponential_with(seed, request, position, pb, (uint32_t)b) / W;
     if (key < b1k) {
       b2k = b1k;
       b2 = b1;
@@ -192,7 +204,7 @@ static int two_level_race(const double* w, int V, uint64_t seed,
     if (b < 0) continue;
     for (int v = b * OR_RACE_BLOCK; v < V && v < (b + 1) * OR_RACE_BLOCK; ++v) {
       if (!(w[v] > 0.0)) continue;
-      double key = oracle_race_exponential(seed, request, position, (uint32_t)v, 2) / w[v];
+      double key = race_exponential_with(seed, request, position, pe, (uint32_t)v) / w[v];
       if (key < yk[pass]) {
         if (pass == 0) {
           y2k = yk[0];
@@ -218,6 +230,14 @@ static int two_level_race(const double* w, int V, uint64_t seed,
     race_out[8] = y[1];
   }
   return y[0];
+}
+
+/* The verification draw (purposes SAMPLE and SAMPLE_IN_BLOCK). */
+static int two_level_race(const double* w, int V, uint64_t seed,
+                          uint64_t request, uint64_t position,
+                          double* race_out) {
+  return two_level_race_with(w, V, seed, request, position, OR_PURPOSE_SAMPLE,
+                             OR_PURPOSE_SAMPLE_IN_BLOCK, race_out);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -477,6 +497,97 @@ int oracle_verify_batch(const void* logits, int logits_dtype,
           race_out ? race_out + (size_t)i * 9 : NULL,
           mode_out ? mode_out + i : NULL);
     }
+    if (status_out) status_out[i] = st;
+    if (st != OR_OK && first == OR_OK) first = st;
+  }
+  return first;
+}
+
+/* ------------------------------------------------------------------------ */
+/* The drafter's producer step (Section 4.2: D-cut reads the drafter's      */
+/* token-level confidences c_{i,t}, Eq. dcut-score; the paper does not      */
+/* define c further).  Reading: for k = 0..K-1, row k of the drafter's      */
+/* logits gives q_k = softmax(l_k / tau), the draft z_{k+1} is drawn from   */
+/* q_k by the two-level race at position pos_base + k + 1 (purposes DRAFT   */
+/* and DRAFT_IN_BLOCK), or is argmax_v l_k (lowest index) when tau == 0,    */
+/* and its confidence is c_{k+1} = q_k(z_{k+1}), with q_k at temperature 1  */
+/* when tau == 0.  Scores as the allocator forms them (Eq. dcut-score):     */
+/* s_0 = 1, s_k = fl32(s_{k-1} * fl32(c_k)).                                */
+/*   logits [K, V] of dtype; z_out [K]; c_out [K] (fp64); s_out [K+1];      */
+/*   m_out, logS_out [K]: each row's max_v l_v / tau' and                   */
+/*   ln sum_v exp(l_v / tau' - m) (tau' = tau, or 1 when tau == 0);         */
+/*   race_out [K][9] or NULL: each row's race record (two_level_race).      */
+/* A row with a NaN, a +inf or no finite entry, or a position past 2^32 - 1 */
+/* makes the request bad: z = -1, c = 0, s_0 = 1 and s_k = 0 for k >= 1.   */
+/* Returns OR_OK or OR_ERR_BAD_INPUT.                                       */
+/* ------------------------------------------------------------------------ */
+int oracle_draft_request(const void* logits, int dtype, int K, int V, double tau,
+                         uint64_t seed, uint64_t request, int64_t pos_base,
+                         int32_t* z_out, double* c_out, float* s_out,
+                         double* m_out, double* logS_out, double* race_out) {
+  const size_t esize = dtype == OR_F32 ? 4 : 2;
+  const double tc = tau > 0.0 ? tau : 1.0;
+  int bad = pos_base < 0 || pos_base + K > (int64_t)0xFFFFFFFF;
+  double* w = (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1));
+  s_out[0] = 1.0f;
+  for (int k = 0; k < K && !bad; ++k) {
+    const void* row = (const char*)logits + (size_t)k * (size_t)V * esize;
+    double m, S;
+    if (!row_softmax_stats(row, dtype, V, tc, &m, &S)) {
+      bad = 1;
+      break;
+    }
+    int z;
+    if (tau == 0.0) {
+      double mx;
+      z = row_argmax(row, dtype, V, &mx);
+      if (race_out)
+        for (int e = 0; e < 9; ++e) race_out[(size_t)k * 9 + e] = -1;
+    } else {
+      for (int v = 0; v < V; ++v) w[v] = row_prob(row, dtype, v, tc, m, S);
+      z = two_level_race_with(w, V, seed, request, (uint64_t)(pos_base + k + 1), OR_PURPOSE_DRAFT,
+                              OR_PURPOSE_DRAFT_IN_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
+    }
+    if (z < 0) {
+      bad = 1;
+      break;
+    }
+    z_out[k] = z;
+    c_out[k] = row_prob(row, dtype, z, tc, m, S);
+    s_out[k + 1] = s_out[k] * (float)c_out[k];
+    m_out[k] = m;
+    logS_out[k] = log(S);
+  }
+  free(w);
+  if (bad) {
+    for (int k = 0; k < K; ++k) {
+      z_out[k] = -1;
+      c_out[k] = 0.0;
+      s_out[k + 1] = 0.0f;
+      m_out[k] = 0.0;
+      logS_out[k] = 0.0;
+    }
+    return OR_ERR_BAD_INPUT;
+  }
+  return OR_OK;
+}
+
+/* The drafter's step for B requests: logits [B, K, V]; outputs per request  */
+/* as in oracle_draft_request (z [B, K], c [B, K], s [B, K+1], m and logS    */
+/* [B, K], race [B, K, 9] or NULL, status [B]).  Returns the first non-OK.   */
+int oracle_draft_batch(const void* logits, int dtype, int B, int K, int V, double tau,
+                       const uint64_t* seeds, const uint64_t* request_ids,
+                       const int64_t* pos_base, int32_t* z_out, double* c_out,
+                       float* s_out, double* m_out, double* logS_out,
+                       double* race_out, int32_t* status_out) {
+  const size_t esize = dtype == OR_F32 ? 4 : 2;
+  int first = OR_OK;
+  for (int i = 0; i < B; ++i) {
+    const size_t r0 = (size_t)i * K;
+    int st = oracle_draft_request((const char*)logits + r0 * (size_t)V * esize, dtype, K, V, tau,
+                                  seeds[i], request_ids[i], pos_base[i], z_out + r0, c_out + r0,
+                                  s_out + (size_t)i * (K + 1), m_out + r0, logS_out + r0,
+                                  race_out ? race_out + r0 * 9 : NULL);
     if (status_out) status_out[i] = st;
     if (st != OR_OK && first == OR_OK) first = st;
   }
