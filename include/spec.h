@@ -16,6 +16,8 @@
  *                  3.1 and 6).
  *   spec_shard_*   spec_verify for a target whose vocabulary is split over
  *                  tensor-parallel ranks (Section 4.4 serves with TP = 8).
+ *   spec_draft     the drafter's side: drafts, their confidences and the
+ *                  D-cut scores from the drafter's logits (Section 4.2).
  *
  * Conventions shared by every entry point
  *   - Pointers marked "device" are CUDA device (or managed) memory of the
@@ -42,6 +44,8 @@
  *   SPEC_PURPOSE_ACCEPT: sub = 0; u = (word0 >> 8) * 2^-24 in [0, 1)
  *   SPEC_PURPOSE_SAMPLE:          sub = b >> 2; block variate E_b from word[b & 3]
  *   SPEC_PURPOSE_SAMPLE_IN_BLOCK: sub = v >> 2; entry variate E'_v from word[v & 3]
+ *   SPEC_PURPOSE_DRAFT, SPEC_PURPOSE_DRAFT_IN_BLOCK: the same two variates
+ *                  for spec_draft's draw of the drafts
  * where a word x gives E = -ln((2 * (x >> 9) + 1) * 2^-24), the midpoint of
  * one of 2^23 cells of (0, 1), so E > 0;
  * so a round replays bit for bit from (seed, request id, position).
@@ -76,6 +80,8 @@ typedef enum { SPEC_BF16 = 0, SPEC_F32 = 1 } spec_dtype;
 #define SPEC_PURPOSE_ACCEPT 1u
 #define SPEC_PURPOSE_SAMPLE 2u
 #define SPEC_PURPOSE_SAMPLE_IN_BLOCK 3u
+#define SPEC_PURPOSE_DRAFT 4u
+#define SPEC_PURPOSE_DRAFT_IN_BLOCK 5u
 
 /* Limits checked on the host (SPEC_ERR_INVALID_ARG beyond them). */
 #define SPEC_MAX_VOCAB (1 << 30)       /* V < 2^30 keeps v >> 2 within 28 bits */
@@ -352,6 +358,45 @@ int spec_shard_finish(const void* races, int S, const void* decisions, int B, in
                       float temperature, const uint64_t* seeds, const uint64_t* request_ids,
                       int32_t* accepted_len_out, int32_t* out_tokens, int32_t* status,
                       cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * spec_draft -- the drafter's producer step: drafts, token-level confidences
+ * and D-cut scores from the drafter's logits in one streaming pass (Section
+ * 4.2: D-cut reads the drafter's confidences c_{i,t} and ranks positions by
+ * s_{i,k} = prod_{t<=k} c_{i,t}, Eq. dcut-score).  For request i and row k
+ * (the drafter's logits for draft z_{k+1}):
+ *   q_k = softmax(l_k / tau') with tau' = tau, or 1 when tau == 0;
+ *   tau  > 0: z_{k+1} is drawn from q_k by the two-level exponential race of
+ *             spec_verify at position pos_base[i] + k + 1, with the variates
+ *             of SPEC_PURPOSE_DRAFT (blocks) and SPEC_PURPOSE_DRAFT_IN_BLOCK
+ *             (entries);
+ *   tau == 0: z_{k+1} = argmax_v l_k[v] (lowest v on ties);
+ *   c_{k+1} = q_k(z_{k+1})  (a reading: the paper does not define c);
+ *   s_0 = 1, s_k = fl32(s_{k-1} * c_k), the scores spec_allocate forms from
+ *   conf.
+ * Arguments
+ *   logits          device [B, K, V] of logits_dtype, rows contiguous.
+ *   seeds, request_ids  device uint64 [B]; pos_base device int64 [B] (the
+ *                   position of the last committed token; pos_base + K < 2^32).
+ *   drafts_out      device int32 [B, K]; conf_out device fp32 [B, K] (the
+ *                   input spec_allocate takes as conf).
+ *   scores_out      device fp32 [B, K+1] or NULL.
+ *   row_stats_out   device fp32 [B*K, 2] or NULL: per row (max_v l/tau',
+ *                   ln sum_v exp(l/tau' - max)).
+ *   status          device int32 [1]: a row with a NaN, a +inf or no finite
+ *                   logit, or a position past 2^32 - 1, sets
+ *                   SPEC_ERR_BAD_INPUT; its request gets drafts -1,
+ *                   confidences 0 and scores (1, 0, ..., 0).
+ *   ws, ws_bytes    device workspace of at least spec_draft_workspace(B, K, V)
+ *                   bytes, 256-byte aligned, zero-filled once before its first
+ *                   use; left zeroed after each call.
+ * Limits: 1 <= B, 1 <= K <= SPEC_MAX_DRAFTS, 1 <= V < SPEC_MAX_VOCAB.
+ * ---------------------------------------------------------------------- */
+size_t spec_draft_workspace(int B, int K, int V);
+int spec_draft(const void* logits, int logits_dtype, int B, int K, int V, float tau,
+               const uint64_t* seeds, const uint64_t* request_ids, const int64_t* pos_base,
+               int32_t* drafts_out, float* conf_out, float* scores_out, float* row_stats_out,
+               int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * spec_profile_stream_pass -- measurement aid.  The next spec_verify call

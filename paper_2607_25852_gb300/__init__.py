@@ -39,7 +39,7 @@ __all__ = [
     "spec_allocate_workspace", "spec_allocate", "spec_verify_workspace", "spec_verify",
     "spec_verify_static", "spec_commit", "spec_profile_stream_pass", "verify_workspace", "library",
     "spec_shard_workspace", "spec_shard_stats", "spec_shard_decide", "spec_shard_sample",
-    "spec_shard_finish", "shard_workspace",
+    "spec_shard_finish", "shard_workspace", "spec_draft_workspace", "spec_draft", "draft_workspace",
 ]
 
 
@@ -170,6 +170,29 @@ def spec_commit(accepted_len, out_tokens, hidden, B, K, packed_tokens_out, commi
         B, K, H, _ptr(packed_tokens_out), _ptr(commit_offsets_out), _ptr(hidden_out),
         _ptr(status), _stream(stream))
     _check(code, "spec_commit")
+
+
+def spec_draft_workspace(B: int, K: int, V: int) -> int:
+    return library().spec_draft_workspace(B, K, V)
+
+
+def draft_workspace(B: int, K: int, V: int, device="cuda"):
+    """A zero-filled workspace for spec_draft."""
+    n = spec_draft_workspace(B, K, V)
+    if n == 0:
+        raise SpecError(ERR_INVALID_ARG, "spec_draft_workspace")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def spec_draft(logits, tau, seeds, request_ids, pos_base, drafts_out, conf_out, ws, scores_out=None,
+               row_stats_out=None, status=None, stream=None):
+    """logits [B, K, V] bf16/fp32 (the drafter's); see spec.h."""
+    B, K, V = logits.shape
+    code = library().spec_draft(
+        _ptr(logits), _dtype(logits), B, K, V, float(tau), _ptr(seeds), _ptr(request_ids), _ptr(pos_base),
+        _ptr(drafts_out), _ptr(conf_out), _ptr(scores_out), _ptr(row_stats_out), _ptr(status), _ptr(ws),
+        _nbytes(ws), _stream(stream))
+    _check(code, "spec_draft")
 
 
 def spec_shard_workspace(B: int, K: int, V_shard: int) -> int:

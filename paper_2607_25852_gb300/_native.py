@@ -27,6 +27,8 @@ SIGNATURES = {
                                 _P, _P, _P, _P, _P, _P, _P]),
     "spec_commit": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
     "spec_profile_stream_pass": (_I, [_P, _P]),
+    "spec_draft_workspace": (_SZ, [_I, _I, _I]),
+    "spec_draft": (_I, [_P, _I, _I, _I, _I, ctypes.c_float, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "spec_shard_workspace": (_SZ, [_I, _I, _I]),
     "spec_shard_stats": (_I, [_P, _I, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, ctypes.c_float, _P, _P,
                               _P, _P, _SZ, _P]),

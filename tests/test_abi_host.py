@@ -126,3 +126,24 @@ def test_shard_workspace_and_argument_errors(lib):
     f = lambda S, t: lib.spec_shard_finish(dummy, S, dummy, 4, 3, 5000, t, dummy, dummy, dummy, dummy,
                                            None, stream)
     assert f(0, 1.0) == 1 and f(2, 0.0) == 0
+
+
+def test_draft_workspace_and_argument_errors(lib):
+    import paper_2607_25852_gb300 as spec
+    assert spec.spec_draft_workspace(0, 4, 100) == 0
+    assert spec.spec_draft_workspace(4, 0, 100) == 0
+    assert spec.spec_draft_workspace(4, 256, 100) == 0
+    n = spec.spec_draft_workspace(64, 16, 201088)
+    assert n > 0 and n % 256 == 0 and n < (1 << 20)
+    dummy = ctypes.c_void_p(16)          # never dereferenced: every call below fails its checks
+    stream = ctypes.c_void_p(0)
+    d = lambda B, K, V, tau, ws=ctypes.c_void_p(256), ws_bytes=1 << 20, dt=0, stats=None: lib.spec_draft(
+        dummy, dt, B, K, V, tau, dummy, dummy, dummy, dummy, dummy, None, stats, None, ws, ws_bytes, stream)
+    assert d(0, 4, 100, 1.0) == 1
+    assert d(4, 0, 100, 1.0) == 1
+    assert d(4, 4, 0, 1.0) == 1
+    assert d(4, 4, 100, -1.0) == 1 and d(4, 4, 100, float("nan")) == 1 and d(4, 4, 100, float("inf")) == 1
+    assert d(4, 4, 100, 1.0, dt=5) == 1
+    assert d(4, 4, 100, 1.0, stats=ctypes.c_void_p(20)) == 1     # row stats not 8-byte aligned
+    assert d(4, 4, 100, 1.0, ws_bytes=8) == 2
+    assert d(4, 4, 100, 1.0, ws=ctypes.c_void_p(264)) == 2

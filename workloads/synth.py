@@ -28,6 +28,9 @@ Recipes (std = standard deviation):
   stress   B=64, K=16, V=201088, bf16 logits ~ N(0, 3^2); q = softmax(target
            + N(0, 1)) stored bf16 [B, K, V]; draft j+1 ~ q_j; temperature 1;
            seed_i = i; hidden rows H=7168 bf16.
+  draft    (make_draft) the drafter's logits [B, K, V] = N(0, 3^2) + N(0, 1),
+           B=64, K=16, V=201088 bf16, tau = 1: the input of the drafter's
+           producer step.
 """
 from dataclasses import dataclass, field
 from typing import Optional
@@ -171,6 +174,38 @@ def make(name: str, *, device="cpu", seed: int = 1234, V: Optional[int] = None,
                   last_tokens=last_tokens.to(device), hidden=hidden,
                   conf=None if conf is None else conf.to(device), extra=extra)
     return wl
+
+
+@dataclass
+class DraftInputs:
+    """Inputs of the drafter's producer step (spec_draft)."""
+    B: int
+    K: int
+    V: int
+    dtype: str
+    tau: float
+    logits: torch.Tensor        # [B, K, V], the drafter's logits for drafts 1..K
+    seeds: torch.Tensor         # int64 [B] (uint64 bits)
+    request_ids: torch.Tensor   # int64 [B]
+    pos_base: torch.Tensor      # int64 [B]
+
+
+def make_draft(B: int = 64, K: int = 16, V: int = 201088, *, tau: float = 1.0, dtype: str = "bf16",
+               std: float = 3.0, device="cpu", seed: int = 4321) -> DraftInputs:
+    """The drafter's logits for one block of K drafts per request: rows of
+    N(0, std^2) (the stress recipe's target rows) plus N(0, 1) noise, the same
+    construction the stress recipe uses for q before its softmax.  B=64, K=16,
+    V=201088 bf16 at tau = 1 by default."""
+    device = torch.device(device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    rng = np.random.default_rng(seed)
+    logits = _normal((B, K, V), std, gen, device)
+    logits += _normal((B, K, V), 1.0, gen, device)
+    return DraftInputs(B=B, K=K, V=V, dtype=dtype, tau=tau, logits=logits.to(_torch_dtype(dtype)),
+                       seeds=torch.arange(B, dtype=torch.int64, device=device) + 77,
+                       request_ids=torch.arange(B, dtype=torch.int64, device=device) + 5000,
+                       pos_base=torch.as_tensor(rng.integers(0, 4096, size=B), dtype=torch.int64).to(device))
 
 
 def pack_rows(full: torch.Tensor, B: int, K: int, depth, row_offsets=None):
