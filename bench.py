@@ -56,6 +56,9 @@ def parse():
     ap.add_argument("--no-graph", action="store_true", help="skip the CUDA-graph replay timing")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--draft", action="store_true",
+                    help="time the drafter's step (spec_draft) on B=64, K=16, V=201088 bf16 drafter logits")
+    ap.add_argument("--tau", type=float, default=1.0, help="draft temperature for --draft")
     ap.add_argument("--shards", type=int, default=1,
                     help="S > 1: time vocabulary-sharded verification with S shards emulated on one GPU")
     return ap.parse_args()
@@ -631,10 +634,75 @@ def run_sharded(args):
     return 0
 
 
+def run_draft(args):
+    """The drafter's producer step (spec_draft) on the draft recipe: drafts,
+    confidences and D-cut scores from B x K rows of drafter logits.  One
+    launch per step; the logits (412 MB) exceed L2, so no flush."""
+    import torch
+    import paper_2607_25852_gb300 as spec
+    import workloads
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    di = workloads.make_draft(device=device, tau=args.tau, B=args.B or 64, V=args.V or 201088)
+    B, K, V = di.B, di.K, di.V
+    ws = spec.draft_workspace(B, K, V, device)
+    z = torch.zeros((B, K), dtype=torch.int32, device=device)
+    c = torch.zeros((B, K), device=device)
+    sc = torch.zeros((B, K + 1), device=device)
+    st = torch.zeros((B * K, 2), device=device)
+    status = torch.zeros(1, dtype=torch.int32, device=device)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        spec.spec_draft(di.logits, di.tau, di.seeds, di.request_ids, di.pos_base, z, c, ws, scores_out=sc,
+                        row_stats_out=st, status=status)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, "device reported an input error"
+    nbytes = di.logits.numel() * di.logits.element_size()
+    flush = None
+    if nbytes < 2 * L2_BYTES:
+        flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=device)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(0) as clocks:
+        for k in range(args.steps):
+            if flush is not None:
+                flush.fill_(k & 0xFF)
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    ms = [a.elapsed_time(b) for a, b in ev]
+    ms_per_step = statistics.mean(ms)
+    peak, peak_kind = measured_peak()
+    achieved = nbytes / (ms_per_step * 1e-3) / 1e9
+    line = {
+        "metric": "drafted positions/s", "value": B * K / (ms_per_step * 1e-3), "unit": "positions/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": di.dtype, "data": "synthetic",
+        "config": {"workload": f"draft: B={B} K={K} V={V} {di.dtype} drafter logits, tau={di.tau}",
+                   "l2": "inputs larger than L2, no flush" if flush is None else "L2 flushed between steps"},
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": None, "kernel": "draft_rows_kernel",
+                     "peak_kind": peak_kind, "algorithmic_bytes_per_launch": nbytes,
+                     "avg_launch_us": round(1e3 * ms_per_step, 2)},
+        "step_ms_p10_p50_p90": [float(np.percentile(ms, q)) for q in (10, 50, 90)],
+        "mean_confidence": float(c.mean().item()),
+        "clocks": clocks.summary(),
+        "gpu_launches": args.steps,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.draft:
+        return run_draft(args)
     if args.shards > 1:
         return run_sharded(args)
     return run_ours(args)
