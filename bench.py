@@ -59,6 +59,9 @@ def parse():
     ap.add_argument("--draft", action="store_true",
                     help="time the drafter's step (spec_draft) on B=64, K=16, V=201088 bf16 drafter logits")
     ap.add_argument("--tau", type=float, default=1.0, help="draft temperature for --draft")
+    ap.add_argument("--round-graph", action="store_true",
+                    help="time a round with the budget chosen on the device (one graph per candidate budget) "
+                         "against the host reading the budget between allocation and verification")
     ap.add_argument("--shards", type=int, default=1,
                     help="S > 1: time vocabulary-sharded verification with S shards emulated on one GPU")
     return ap.parse_args()
@@ -697,10 +700,126 @@ def run_draft(args):
     return 0
 
 
+def run_round_graph(args):
+    """A round of allocate -> verify -> commit on the stress workload with the
+    D-cut ratios 1/4..1 and the piecewise-linear cost 1 + 0.004 max(0, T - 256).
+    (a) host-driven: the host reads T* after spec_allocate, then launches the
+    graph of verify + commit captured for that shape; (b) device-selected: one
+    host-launched graph allocates and tail-launches the graph of T*.  The
+    packed logits of every candidate shape are prepared once beforehand (the
+    target forward, which would write them, is not part of this library)."""
+    import torch
+    import paper_2607_25852_gb300 as spec
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    wl = make_inputs(args, 0, device)
+    B, K, V = wl.B, wl.K, wl.V
+    Ts = spec.spec_budget_from_ratios(B, K, [1, 1, 3, 1], [4, 2, 4, 1])
+    costs = [1.0 + 0.004 * max(0, T - 256) for T in Ts]
+    st = Step(wl, device)
+    st.ratios, st.costs = Ts, costs
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        st.spec.spec_allocate(wl.conf, Ts, costs, wl.last_tokens, wl.drafts, wl.pos_base, st.depth, st.row_off,
+                              st.ptok, st.ppos, st.chosen, st.util, st.status)
+    s.synchronize()
+    T_star = int(st.chosen.item())
+    m_star = Ts.index(T_star)
+    lg = []
+    for T in Ts:
+        buf = torch.zeros((T, V), dtype=wl.logits.dtype, device=device)
+        with torch.cuda.stream(s):
+            spec.spec_pack_rows(wl.logits, B, K, st.row_off, buf, status=st.status)  # this allocation's packing
+        lg.append(buf)
+    hid = torch.zeros((T_star, wl.H), dtype=torch.bfloat16, device=device)
+    with torch.cuda.stream(s):
+        spec.spec_pack_rows(wl.hidden, B, K, st.row_off, hid, status=st.status)
+    s.synchronize()
+
+    def after(m):
+        spec.spec_verify(lg[m], wl.drafts, wl.q, B, K, V, wl.temperature, wl.seeds, wl.request_ids, wl.pos_base,
+                         st.acc, st.tok, st.ws, row_offsets=st.row_off, depth=st.depth, status=st.status)
+        spec.spec_commit(st.acc, st.tok, hid if m == m_star else None, B, K, st.ctok, st.coff,
+                         st.hout if m == m_star else None, row_offsets=st.row_off, status=st.status)
+
+    def allocate():
+        spec.spec_allocate(wl.conf, Ts, costs, wl.last_tokens, wl.drafts, wl.pos_base, st.depth, st.row_off,
+                           st.ptok, st.ppos, st.chosen, st.util, st.status)
+
+    children = []
+    launched = torch.zeros(1, dtype=torch.int32, device=device)
+    with torch.cuda.stream(s):
+        for m in range(len(Ts)):
+            spec.spec_graph_begin_capture(s)
+            after(m)
+            children.append(spec.spec_graph_end_capture(s, device_launch=True))
+        spec.spec_graph_begin_capture(s)
+        allocate()
+        spec.spec_select_round(st.chosen, Ts, children, launched, st.status)
+        parent = spec.spec_graph_end_capture(s, device_launch=False)
+
+    def host_round():
+        with torch.cuda.stream(s):
+            allocate()
+            s.synchronize()
+            m = Ts.index(int(st.chosen.item()))
+            spec.spec_graph_launch(children[m], s)
+            s.synchronize()
+
+    def device_round():
+        spec.spec_graph_launch(parent, s)
+        s.synchronize()
+
+    def timed(fn, n):
+        for _ in range(max(args.warmup, 3)):
+            fn()
+        t0 = time.perf_counter()
+        for _ in range(n):
+            fn()
+        return (time.perf_counter() - t0) / n
+
+    n = args.steps
+    host_s = timed(host_round, n)
+    dev_s = timed(device_round, n)
+    # back to back (no host wait between rounds): device time per round
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clocks:
+        a.record(s)
+        for _ in range(n):
+            spec.spec_graph_launch(parent, s)
+        b.record(s)
+        s.synchronize()
+    chain_ms = a.elapsed_time(b) / n
+    assert int(st.status.item()) == 0 and int(launched.item()) == m_star
+    for g in children + [parent]:
+        spec.spec_graph_destroy(g)
+    line = {
+        "metric": "round latency (allocate + verify + commit)", "value": dev_s * 1e6, "unit": "us",
+        "n_gpus": 1, "steps": n, "warmup": args.warmup, "ms_per_step": dev_s * 1e3, "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": f"{wl.name}: B={B} K={K} V={V} {wl.dtype} logits, t={wl.temperature}; D-cut ratios "
+                               f"1/4..1, cost 1 + 0.004 max(0, T - 256): T* = {T_star} of {Ts}",
+                   "candidate_graphs": len(Ts)},
+        "host_driven_round_us": round(host_s * 1e6, 2),
+        "device_selected_round_us": round(dev_s * 1e6, 2),
+        "device_selected_back_to_back_us": round(chain_ms * 1e3, 2),
+        "saved_per_round_us": round((host_s - dev_s) * 1e6, 2),
+        "how": "wall clock per round with a host wait at its end; back to back: CUDA events over consecutive "
+               "parent-graph launches",
+        "clocks": clocks.summary(),
+        "gpu_launches": 6 * n,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.round_graph:
+        return run_round_graph(args)
     if args.draft:
         return run_draft(args)
     if args.shards > 1:

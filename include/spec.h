@@ -18,6 +18,9 @@
  *                  tensor-parallel ranks (Section 4.4 serves with TP = 8).
  *   spec_draft     the drafter's side: drafts, their confidences and the
  *                  D-cut scores from the drafter's logits (Section 4.2).
+ *   spec_graph_*, spec_select_round
+ *                  a round per candidate budget as CUDA graphs, the budget
+ *                  chosen on the device (Section 4.3).
  *
  * Conventions shared by every entry point
  *   - Pointers marked "device" are CUDA device (or managed) memory of the
@@ -397,6 +400,57 @@ int spec_draft(const void* logits, int logits_dtype, int B, int K, int V, float 
                const uint64_t* seeds, const uint64_t* request_ids, const int64_t* pos_base,
                int32_t* drafts_out, float* conf_out, float* scores_out, float* row_stats_out,
                int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * A whole round per candidate budget as CUDA graphs, the budget chosen on the
+ * device (Section 4.3: the reachable verification shapes form a small finite
+ * set, so a graph can be captured per (B, rho), and budget selection should
+ * leave the critical path instead of synchronising drafting and
+ * verification).  Recipe:
+ *   1. per candidate T_m: spec_graph_begin_capture(s); enqueue on s what
+ *      follows the allocation at that shape (the target forward over T_m
+ *      packed rows -- spec_pack_rows stands in for it -- then spec_verify and
+ *      spec_commit); spec_graph_end_capture(s, 1, &g[m]);
+ *   2. spec_graph_begin_capture(s); spec_allocate(...);
+ *      spec_select_round(chosen_T, M, cand_T, g, ...);
+ *      spec_graph_end_capture(s, 0, &parent);
+ *   3. every round: spec_graph_launch(parent, s).  The selector kernel reads
+ *      T* on the device and tail-launches g[m] with cand_T[m] == T*: the
+ *      round needs no host round trip between the budget choice and the
+ *      verification.  Work enqueued on s after the parent waits for the
+ *      tail-launched graph too.
+ * Graph handles are opaque (cudaGraphExec_t); instantiating a graph allocates
+ * what the CUDA driver needs for it (the one exception to "the library never
+ * allocates device memory"), released by spec_graph_destroy.
+ * ---------------------------------------------------------------------- */
+/* Begin capturing `stream` (relaxed capture mode; not the legacy stream). */
+int spec_graph_begin_capture(cudaStream_t stream);
+/* End the capture and instantiate it; device_launch != 0 instantiates for
+ * launch from the device (and uploads it).  *exec_out: the graph handle. */
+int spec_graph_end_capture(cudaStream_t stream, int device_launch, void** exec_out);
+int spec_graph_launch(void* exec, cudaStream_t stream);
+int spec_graph_destroy(void* exec);
+
+/* spec_select_round -- one thread on `stream`: reads *chosen_T (device, as
+ * spec_allocate writes it), finds m with cand_T[m] == T*, tail-launches
+ * graphs[m] (instantiated with device_launch) and writes m to *launched_out
+ * (device int32, or NULL).  Must be captured into a host-launched graph (the
+ * device runtime launches graphs only from kernels that run in a graph).  A
+ * T* that is not in cand_T sets SPEC_ERR_BAD_INPUT and launches nothing.
+ *   cand_T, graphs  host [M], 1 <= M <= SPEC_MAX_CANDIDATES. */
+int spec_select_round(const int32_t* chosen_T, int M, const int32_t* cand_T, void* const* graphs,
+                      int32_t* launched_out, int32_t* status, cudaStream_t stream);
+
+/* spec_pack_rows -- the packed layout of an allocation applied to a
+ * full-depth buffer: dst row row_offsets[i] + j = src row i(K+1) + j for
+ * j <= n_i (Section 4.2 "Packing and correctness"), rows of row_bytes bytes.
+ * Stands in for a target forward that writes its outputs in packed order.
+ *   src             device [B(K+1), row_bytes]; dst device [R_dst, row_bytes]
+ *                   (R_dst >= row_offsets[B]; rows past it are not written).
+ *   row_offsets     device int32 [B+1] from spec_allocate.
+ * A row whose offset within its request exceeds K sets SPEC_ERR_BAD_INPUT. */
+int spec_pack_rows(const void* src, size_t row_bytes, int B, int K, const int32_t* row_offsets,
+                   void* dst, int R_dst, int32_t* status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * spec_profile_stream_pass -- measurement aid.  The next spec_verify call

@@ -40,6 +40,8 @@ __all__ = [
     "spec_verify_static", "spec_commit", "spec_profile_stream_pass", "verify_workspace", "library",
     "spec_shard_workspace", "spec_shard_stats", "spec_shard_decide", "spec_shard_sample",
     "spec_shard_finish", "shard_workspace", "spec_draft_workspace", "spec_draft", "draft_workspace",
+    "spec_graph_begin_capture", "spec_graph_end_capture", "spec_graph_launch", "spec_graph_destroy",
+    "spec_select_round", "spec_pack_rows",
 ]
 
 
@@ -170,6 +172,47 @@ def spec_commit(accepted_len, out_tokens, hidden, B, K, packed_tokens_out, commi
         B, K, H, _ptr(packed_tokens_out), _ptr(commit_offsets_out), _ptr(hidden_out),
         _ptr(status), _stream(stream))
     _check(code, "spec_commit")
+
+
+def spec_graph_begin_capture(stream):
+    """Begin capturing `stream` (a torch.cuda.Stream, not the default stream)."""
+    _check(library().spec_graph_begin_capture(_stream(stream)), "spec_graph_begin_capture")
+
+
+def spec_graph_end_capture(stream, device_launch: bool):
+    """End the capture; returns the instantiated graph handle (an int)."""
+    out = ctypes.c_void_p()
+    _check(library().spec_graph_end_capture(_stream(stream), int(bool(device_launch)), ctypes.byref(out)),
+           "spec_graph_end_capture")
+    return out.value
+
+
+def spec_graph_launch(graph, stream=None):
+    _check(library().spec_graph_launch(ctypes.c_void_p(graph), _stream(stream)), "spec_graph_launch")
+
+
+def spec_graph_destroy(graph):
+    _check(library().spec_graph_destroy(ctypes.c_void_p(graph)), "spec_graph_destroy")
+
+
+def spec_select_round(chosen_T, cand_T, graphs, launched_out=None, status=None, stream=None):
+    """chosen_T: device int32 [1]; cand_T: host ints [M]; graphs: handles [M]."""
+    M = len(cand_T)
+    if len(graphs) != M:
+        raise SpecError(ERR_INVALID_ARG, "spec_select_round: one graph per candidate")
+    Ts = (ctypes.c_int32 * M)(*[int(t) for t in cand_T])
+    gs = (ctypes.c_void_p * M)(*graphs)
+    _check(library().spec_select_round(_ptr(chosen_T), M, Ts, gs, _ptr(launched_out), _ptr(status),
+                                       _stream(stream)), "spec_select_round")
+
+
+def spec_pack_rows(src, B, K, row_offsets, dst, status=None, stream=None):
+    """src [B(K+1), ...], dst [R_dst, ...] with the same row size."""
+    row_bytes = src[0].numel() * src.element_size()
+    if dst[0].numel() * dst.element_size() != row_bytes:
+        raise SpecError(ERR_INVALID_ARG, "spec_pack_rows: row sizes differ")
+    _check(library().spec_pack_rows(_ptr(src), row_bytes, B, K, _ptr(row_offsets), _ptr(dst), dst.shape[0],
+                                    _ptr(status), _stream(stream)), "spec_pack_rows")
 
 
 def spec_draft_workspace(B: int, K: int, V: int) -> int:

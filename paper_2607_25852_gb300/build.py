@@ -37,9 +37,15 @@ def up_to_date() -> bool:
     return all(os.path.getmtime(d) <= t for d in _deps())
 
 
+# Translation units that call the device runtime (device-side cudaGraphLaunch):
+# compiled as relocatable device code, device-linked with libcudadevrt.
+RDC_SOURCES = {"round.cu"}
+
+
 def _compile(src, extra):
     obj = os.path.join(BUILD, os.path.basename(src) + ".o")
-    cmd = [NVCC, *ARCH, *FLAGS, *extra, "-c", src, "-o", obj]
+    rdc = ["-rdc=true"] if os.path.basename(src) in RDC_SOURCES else []
+    cmd = [NVCC, *ARCH, *FLAGS, *rdc, *extra, "-c", src, "-o", obj]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"nvcc failed for {src}:\n{res.stdout}\n{res.stderr}")
@@ -58,7 +64,7 @@ def build(force: bool = False, verbose: bool = False, extra=()) -> str:
             if log.strip():
                 print(log)
     tmp = LIBRARY + ".tmp"
-    cmd = [NVCC, *ARCH, "-shared", "-o", tmp, *[o for o, _ in results]]
+    cmd = [NVCC, *ARCH, "-shared", "-rdc=true", "-o", tmp, *[o for o, _ in results], "-lcudadevrt"]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
