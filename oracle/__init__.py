@@ -66,6 +66,10 @@ def _declare(lib):
     lib.oracle_draft_batch.argtypes = [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                        ctypes.c_double, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
     lib.oracle_draft_batch.restype = ctypes.c_int
+    lib.oracle_markov_request.argtypes = [_P, ctypes.c_int, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                          ctypes.c_int32, ctypes.c_double, ctypes.c_uint64, ctypes.c_uint64,
+                                          ctypes.c_int64, _P, _P, _P, _P, _P, _P]
+    lib.oracle_markov_request.restype = ctypes.c_int
     lib.oracle_budget.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, ctypes.c_int64]
     lib.oracle_budget.restype = ctypes.c_int
     lib.oracle_allocate.argtypes = [
@@ -243,6 +247,47 @@ def draft_batch(logits, tau, seeds, request_ids, pos_base):
         _ptr(logits), _dtype_code(logits), B, K, V, float(tau), _ptr(seeds), _ptr(request_ids),
         _ptr(pos_base), _ptr(out["z"]), _ptr(out["c"]), _ptr(out["s"]), _ptr(out["m"]),
         _ptr(out["logS"]), _ptr(out["race"]), _ptr(out["status"]))
+    return out
+
+
+def markov_batch(U, W1, W2, x0, tau, seeds, request_ids, pos_base, requests=None, threads=1):
+    """The Markov head's sequential draw (oracle_markov_request) for each
+    request: U [B, K, V] base logits; W1 [V, r] and W2 [r, V] as bf16 bits
+    (uint16); x0 [B] the last committed tokens.  ``requests`` restricts the
+    work to some requests (the others keep their fill values); ``threads``
+    runs requests side by side (each call is independent)."""
+    U = _c(U)
+    B, K, V = U.shape
+    W1 = _c(W1, np.uint16)
+    W2 = _c(W2, np.uint16)
+    r = W1.shape[1]
+    assert W1.shape == (V, r) and W2.shape == (r, V)
+    x0 = _c(x0, np.int32)
+    seeds = _c(seeds, np.uint64)
+    request_ids = _c(request_ids, np.uint64)
+    pos_base = _c(pos_base, np.int64)
+    out = dict(z=np.full((B, K), -1, np.int32), c=np.zeros((B, K), np.float64),
+               s=np.zeros((B, K + 1), np.float32), m=np.zeros((B, K), np.float64),
+               logS=np.zeros((B, K), np.float64), race=np.zeros((B, K, 9), np.float64),
+               status=np.zeros(B, np.int32))
+    lib = load()
+
+    def one(i):
+        row = U[i]
+        out["status"][i] = lib.oracle_markov_request(
+            _ptr(row), _dtype_code(U), _ptr(W1), _ptr(W2), K, V, r, int(x0[i]), float(tau), int(seeds[i]),
+            int(request_ids[i]), int(pos_base[i]), out["z"][i].ctypes.data, out["c"][i].ctypes.data,
+            out["s"][i].ctypes.data, out["m"][i].ctypes.data, out["logS"][i].ctypes.data,
+            out["race"][i].ctypes.data)
+
+    idx = list(range(B)) if requests is None else list(requests)
+    if threads > 1:
+        import concurrent.futures as cf
+        with cf.ThreadPoolExecutor(threads) as ex:
+            list(ex.map(one, idx))
+    else:
+        for i in idx:
+            one(i)
     return out
 
 

@@ -572,6 +572,93 @@ int oracle_draft_request(const void* logits, int dtype, int K, int V, double tau
   return OR_OK;
 }
 
+/* ------------------------------------------------------------------------ */
+/* The Markov head's sequential draw (Section 3.2, Eq. dspark-markov, after   */
+/* the block factorisation Eq. ar-factorization): the drafter's base logits  */
+/* U_k of each position get the first-order bias b_k = W1[x_{k-1}] W2 of the */
+/* previously drawn token (x_0 the last committed token), and               */
+/* q_k = softmax((U_k + b_k) / tau').  Draws, confidences, scores and the    */
+/* bad-input rule as in oracle_draft_request, position by position.          */
+/*   U [K, V] of dtype; W1 [V, r] and W2 [r, V] bf16 bits (uint16).          */
+/* ------------------------------------------------------------------------ */
+static double bf16_value(uint16_t h) {
+  uint32_t w = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &w, 4);
+  return (double)f;
+}
+
+int oracle_markov_request(const void* U, int dtype, const uint16_t* W1, const uint16_t* W2, int K, int V,
+                          int r, int32_t x0, double tau, uint64_t seed, uint64_t request,
+                          int64_t pos_base, int32_t* z_out, double* c_out, float* s_out,
+                          double* m_out, double* logS_out, double* race_out) {
+  const size_t esize = dtype == OR_F32 ? 4 : 2;
+  const double tc = tau > 0.0 ? tau : 1.0;
+  int bad = pos_base < 0 || pos_base + K > (int64_t)0xFFFFFFFF || x0 < 0 || x0 >= V;
+  double* l = (double*)malloc(sizeof(double) * (size_t)V);
+  double* w = (double*)malloc(sizeof(double) * (size_t)V);
+  s_out[0] = 1.0f;
+  int prev = x0;
+  for (int k = 0; k < K && !bad; ++k) {
+    const void* urow = (const char*)U + (size_t)k * (size_t)V * esize;
+    /* l = U_k + W1[prev] W2, in double */
+    for (int v = 0; v < V; ++v) {
+      double b = 0.0;
+      for (int j = 0; j < r; ++j) b += bf16_value(W1[(size_t)prev * r + j]) * bf16_value(W2[(size_t)j * V + v]);
+      l[v] = load_value(urow, dtype, v) + b;
+      if (isnan(l[v]) || l[v] == INFINITY) bad = 1;
+    }
+    if (bad) break;
+    double m = -INFINITY;
+    for (int v = 0; v < V; ++v)
+      if (l[v] / tc > m) m = l[v] / tc;
+    if (m == -INFINITY) {
+      bad = 1;
+      break;
+    }
+    double S = 0.0;
+    for (int v = 0; v < V; ++v) S += exp(l[v] / tc - m);
+    int z = -1;
+    if (tau == 0.0) {
+      double best = -INFINITY;
+      for (int v = 0; v < V; ++v)
+        if (z < 0 || l[v] > best) {
+          z = v;
+          best = l[v];
+        }
+      if (race_out)
+        for (int e = 0; e < 9; ++e) race_out[(size_t)k * 9 + e] = -1;
+    } else {
+      for (int v = 0; v < V; ++v) w[v] = exp(l[v] / tc - m) / S;
+      z = two_level_race_with(w, V, seed, request, (uint64_t)(pos_base + k + 1), OR_PURPOSE_DRAFT,
+                              OR_PURPOSE_DRAFT_IN_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
+    }
+    if (z < 0) {
+      bad = 1;
+      break;
+    }
+    z_out[k] = z;
+    c_out[k] = exp(l[z] / tc - m) / S;
+    s_out[k + 1] = s_out[k] * (float)c_out[k];
+    m_out[k] = m;
+    logS_out[k] = log(S);
+    prev = z;
+  }
+  free(l);
+  free(w);
+  if (bad) {
+    for (int k = 0; k < K; ++k) {
+      z_out[k] = -1;
+      c_out[k] = 0.0;
+      s_out[k + 1] = 0.0f;
+      m_out[k] = 0.0;
+      logS_out[k] = 0.0;
+    }
+    return OR_ERR_BAD_INPUT;
+  }
+  return OR_OK;
+}
+
 /* The drafter's step for B requests: logits [B, K, V]; outputs per request  */
 /* as in oracle_draft_request (z [B, K], c [B, K], s [B, K+1], m and logS    */
 /* [B, K], race [B, K, 9] or NULL, status [B]).  Returns the first non-OK.   */
