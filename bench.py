@@ -59,6 +59,9 @@ def parse():
     ap.add_argument("--draft", action="store_true",
                     help="time the drafter's step (spec_draft) on B=64, K=16, V=201088 bf16 drafter logits")
     ap.add_argument("--tau", type=float, default=1.0, help="draft temperature for --draft")
+    ap.add_argument("--markov", action="store_true",
+                    help="time the Markov head's sequential draw: B=64 requests, a block of K=7 drafts, "
+                         "V=201088, rank r=256")
     ap.add_argument("--round-graph", action="store_true",
                     help="time a round with the budget chosen on the device (one graph per candidate budget) "
                          "against the host reading the budget between allocation and verification")
@@ -700,6 +703,71 @@ def run_draft(args):
     return 0
 
 
+def run_markov(args):
+    """The Markov head's sequential draw (spec_markov_draft): per position, a
+    [B, r] x [r, V] bias contraction on the tensor cores fused with the draw.
+    Synthetic base logits N(0, 3^2) and factors N(0, 0.2^2), bf16."""
+    import torch
+    import paper_2607_25852_gb300 as spec
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    B, K, V, r = args.B or 64, 7, args.V or 201088, 256
+    g = torch.Generator(device=device)
+    g.manual_seed(1234)
+    U = (torch.randn((B, K, V), generator=g, device=device) * 3.0).to(torch.bfloat16)
+    W1 = (torch.randn((V, r), generator=g, device=device) * 0.2).to(torch.bfloat16)
+    W2T = (torch.randn((V, r), generator=g, device=device) * 0.2).to(torch.bfloat16)
+    x0 = torch.randint(0, V, (B,), generator=g, device=device, dtype=torch.int32)
+    seeds = torch.arange(B, dtype=torch.int64, device=device) + 11
+    rids = torch.arange(B, dtype=torch.int64, device=device) + 7000
+    pos = torch.randint(0, 4096, (B,), generator=g, device=device, dtype=torch.int64)
+    ws = spec.markov_workspace(B, K, V, r, device)
+    z = torch.zeros((B, K), dtype=torch.int32, device=device)
+    c = torch.zeros((B, K), device=device)
+    sc = torch.zeros((B, K + 1), device=device)
+    status = torch.zeros(1, dtype=torch.int32, device=device)
+    stream = torch.cuda.current_stream()
+    tau = args.tau
+
+    def step():
+        spec.spec_markov_draft(U, W1, W2T, x0, tau, seeds, rids, pos, z, c, ws, scores_out=sc, status=status)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, "device reported an error"
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(0) as clocks:
+        for k in range(args.steps):
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    peak, peak_kind = measured_peak()
+    # per position: the whole W2 (V x r) and the position's base logits (B x V)
+    per_pos = V * r * 2 + B * V * 2
+    achieved = per_pos * K / (ms * 1e-3) / 1e9
+    flops = 2.0 * B * r * V * K
+    line = {
+        "metric": "drafted positions/s (Markov head)", "value": B * K / (ms * 1e-3), "unit": "positions/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"markov: B={B} requests, K={K} drafts (block of 8), V={V}, r={r}, tau={tau}",
+                   "l2": "W2 (%.0f MB) is read once per position; it fits in L2 between positions" % (V * r * 2 / 1e6)},
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": None, "kernel": "markov_bias_kernel + markov_pick_kernel",
+                     "peak_kind": peak_kind, "algorithmic_bytes_per_position": per_pos,
+                     "avg_step_us": round(ms * 1e3, 2)},
+        "tensor_tflops": round(flops / (ms * 1e-3) / 1e12, 2),
+        "per_position_us": round(ms * 1e3 / K, 2),
+        "clocks": clocks.summary(),
+        "gpu_launches": (1 + 2 * K) * args.steps,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_round_graph(args):
     """A round of allocate -> verify -> commit on the stress workload with the
     D-cut ratios 1/4..1 and the piecewise-linear cost 1 + 0.004 max(0, T - 256).
@@ -820,6 +888,8 @@ def main():
         return run_reference(args)
     if args.round_graph:
         return run_round_graph(args)
+    if args.markov:
+        return run_markov(args)
     if args.draft:
         return run_draft(args)
     if args.shards > 1:

@@ -18,6 +18,9 @@
  *                  tensor-parallel ranks (Section 4.4 serves with TP = 8).
  *   spec_draft     the drafter's side: drafts, their confidences and the
  *                  D-cut scores from the drafter's logits (Section 4.2).
+ *   spec_markov_draft
+ *                  the Markov head's sequential draw over a block (Section
+ *                  3.2): a tensor-core contraction per position.
  *   spec_graph_*, spec_select_round
  *                  a round per candidate budget as CUDA graphs, the budget
  *                  chosen on the device (Section 4.3).
@@ -400,6 +403,35 @@ int spec_draft(const void* logits, int logits_dtype, int B, int K, int V, float 
                const uint64_t* seeds, const uint64_t* request_ids, const int64_t* pos_base,
                int32_t* drafts_out, float* conf_out, float* scores_out, float* row_stats_out,
                int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * spec_markov_draft -- the Markov head's sequential draw (Section 3.2,
+ * Eq. dspark-markov; the block factorisation Eq. ar-factorization): for
+ * k = 0..K-1, with x_0 the last committed token,
+ *   b_k = W1[x_k] W2,  q_k = softmax((U_k + b_k) / tau')  (tau' = tau, or 1),
+ *   x_{k+1} ~ q_k by the two-level race at position pos_base + k + 1
+ *   (purposes SPEC_PURPOSE_DRAFT / _IN_BLOCK), argmax at tau == 0;
+ *   c_{k+1} = q_k(x_{k+1}); scores as spec_draft.
+ * The bias of all B requests is one [B, r] x [r, V] contraction per position,
+ * run on the tensor cores (tcgen05, fp32 accumulation): q, c and the row
+ * statistics carry its rounding (relative errors of order r * 2^-24 on the
+ * bias).
+ *   U               device bf16 [B, K, V]: the backbone's base logits.
+ *   W1              device bf16 [V, r]; W2T device bf16 [V, r], W2 stored
+ *                   transposed (row v = column v of W2), 16-byte aligned.
+ *   r               the factorisation's rank: a multiple of 64, 64..256.
+ *   x0              device int32 [B]: each request's last committed token.
+ *   B <= 128; other arguments and the bad-input rule as spec_draft (an x0
+ *   outside [0, V) also makes the request bad).
+ *   ws, ws_bytes    spec_markov_workspace(B, K, V, r) bytes, 256-aligned, no
+ *                   zeroing needed.
+ * ---------------------------------------------------------------------- */
+size_t spec_markov_workspace(int B, int K, int V, int r);
+int spec_markov_draft(const void* U, int u_dtype, const void* W1, const void* W2T, int r,
+                      const int32_t* x0, int B, int K, int V, float tau, const uint64_t* seeds,
+                      const uint64_t* request_ids, const int64_t* pos_base, int32_t* drafts_out,
+                      float* conf_out, float* scores_out, float* row_stats_out, int32_t* status,
+                      void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * A whole round per candidate budget as CUDA graphs, the budget chosen on the

@@ -41,7 +41,7 @@ __all__ = [
     "spec_shard_workspace", "spec_shard_stats", "spec_shard_decide", "spec_shard_sample",
     "spec_shard_finish", "shard_workspace", "spec_draft_workspace", "spec_draft", "draft_workspace",
     "spec_graph_begin_capture", "spec_graph_end_capture", "spec_graph_launch", "spec_graph_destroy",
-    "spec_select_round", "spec_pack_rows",
+    "spec_select_round", "spec_pack_rows", "spec_markov_workspace", "spec_markov_draft", "markov_workspace",
 ]
 
 
@@ -172,6 +172,29 @@ def spec_commit(accepted_len, out_tokens, hidden, B, K, packed_tokens_out, commi
         B, K, H, _ptr(packed_tokens_out), _ptr(commit_offsets_out), _ptr(hidden_out),
         _ptr(status), _stream(stream))
     _check(code, "spec_commit")
+
+
+def spec_markov_workspace(B: int, K: int, V: int, r: int) -> int:
+    return library().spec_markov_workspace(B, K, V, r)
+
+
+def markov_workspace(B: int, K: int, V: int, r: int, device="cuda"):
+    n = spec_markov_workspace(B, K, V, r)
+    if n == 0:
+        raise SpecError(ERR_INVALID_ARG, "spec_markov_workspace")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def spec_markov_draft(U, W1, W2T, x0, tau, seeds, request_ids, pos_base, drafts_out, conf_out, ws,
+                      scores_out=None, row_stats_out=None, status=None, stream=None):
+    """U [B, K, V] bf16; W1 and W2T [V, r] bf16 (W2T = W2 transposed); x0 [B] int32."""
+    B, K, V = U.shape
+    r = W1.shape[1]
+    code = library().spec_markov_draft(
+        _ptr(U), _dtype(U), _ptr(W1), _ptr(W2T), r, _ptr(x0), B, K, V, float(tau), _ptr(seeds),
+        _ptr(request_ids), _ptr(pos_base), _ptr(drafts_out), _ptr(conf_out), _ptr(scores_out),
+        _ptr(row_stats_out), _ptr(status), _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(code, "spec_markov_draft")
 
 
 def spec_graph_begin_capture(stream):

@@ -29,6 +29,9 @@ SIGNATURES = {
     "spec_profile_stream_pass": (_I, [_P, _P]),
     "spec_draft_workspace": (_SZ, [_I, _I, _I]),
     "spec_draft": (_I, [_P, _I, _I, _I, _I, ctypes.c_float, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "spec_markov_workspace": (_SZ, [_I, _I, _I, _I]),
+    "spec_markov_draft": (_I, [_P, _I, _P, _P, _I, _P, _I, _I, _I, ctypes.c_float, _P, _P, _P, _P, _P, _P, _P,
+                               _P, _P, _SZ, _P]),
     "spec_graph_begin_capture": (_I, [_P]),
     "spec_graph_end_capture": (_I, [_P, _I, ctypes.POINTER(ctypes.c_void_p)]),
     "spec_graph_launch": (_I, [_P, _P]),

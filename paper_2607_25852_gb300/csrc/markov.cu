@@ -1,0 +1,707 @@
+// markov.cu -- the Markov head's sequential draw on sm_103a (arxiv
+// 2607.25852, Section 3.2, Eq. dspark-markov: each position's base logits
+// U_k get the first-order bias b_k = W1[x_{k-1}] W2 of the previously drawn
+// token, q_k = softmax(U_k + b_k); the block distribution factorises over the
+// positions, Eq. ar-factorization).
+//
+// Per position k, for all B requests at once, the bias is the dense
+// contraction E_k W2 with E_k = W1[x_{k-1}] ([B, r] x [r, V]): it runs on the
+// 5th-generation tensor cores.
+//
+//   markov_bias_kernel  persistent, one CTA per SM.  Warp 0 loads by TMA the
+//                       operand E_k (128 x r, requests padded with zero rows)
+//                       once and then tiles of W2^T (128 vocabulary rows x r,
+//                       128-byte swizzle), double-buffered.  Warp 1 issues
+//                       tcgen05.mma (M = 128, N = 128, K = 16, bf16 -> fp32)
+//                       into two TMEM accumulators.  The epilogue warps read
+//                       the accumulator rows (tcgen05.ld, one request per
+//                       thread), add U_k, and per race block of 256 entries
+//                       form the block's max and sum, its level-1 race key
+//                       (or its argmax at tau = 0) and the row's softmax
+//                       statistics.  Each CTA writes one partial per request.
+//   markov_pick_kernel  one CTA per request: merges the partials, recomputes
+//                       the winning block's 256 logits and draws inside it
+//                       (level 2), writes the draft, its confidence and the
+//                       row statistics, and gathers W1 at the draft into E for
+//                       the next position.
+//
+// Every mbarrier wait is bounded (about a second): a wait that gives up sets
+// SPEC_ERR_TIMEOUT, the kernel stops issuing work, waits (bounded) for what
+// it issued, frees its TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+
+#include "verify_common.cuh"
+
+namespace spec {
+
+constexpr int kMkRows = 128;        // MMA M: request rows (rows >= B are zero)
+constexpr int kMkTile = 128;        // MMA N: vocabulary rows of W2^T per tile
+constexpr int kMkAtomK = 64;        // bf16 along K per 128-byte swizzle atom
+constexpr int kMkAtomBytes = 128 * 128;  // one atom of 128 rows x 128 bytes
+constexpr int kMkThreads = 192;     // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kMkMaxR = 256;
+constexpr int kMkTmemCols = 256;    // two accumulators of kMkTile fp32 columns
+constexpr int kPickThreads = 256;
+
+struct alignas(16) MkPartial {
+  float m, s;     // softmax statistics of the CTA's columns (s relative to fl(m*c2))
+  float L;        // tau > 0: best block's log2 E - log2 sum; tau = 0: the max
+  int32_t idx;    // tau > 0: best block; tau = 0: lowest argmax (INT_MAX: none)
+  float M;        // tau > 0: best block's max
+  int32_t flags;  // bit0: NaN or +inf
+  int32_t pad[2];
+};
+
+struct MarkovLaunch {
+  const __nv_bfloat16* U;    // [B, K, V]
+  const __nv_bfloat16* W1;   // [V, r]
+  const __nv_bfloat16* W2T;  // [V, r]: row v = column v of W2
+  int r, B, K, V, step;
+  float tau, c2, inv_t;
+  const uint64_t* seeds;
+  const uint64_t* request_ids;
+  const int64_t* pos_base;
+  const int32_t* x0;
+  __nv_bfloat16* E;  // [128, r]: W1 at the previous drafts
+  MkPartial* part;   // [B][G]
+  int G;
+  uint32_t* req_bad;  // [B]
+  int32_t* drafts;
+  float* conf;
+  float* scores;
+  float* row_stats;
+  int32_t* status;
+  bool u_vec;
+};
+
+// ---------------------------------------------------------------------------
+// PTX wrappers: mbarrier, TMA, tcgen05
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Wait for the phase with parity `parity`; false (and SPEC_ERR_TIMEOUT) after
+// about a second.
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 255u && global_ns() - t0 > 1000000000ull) {
+      report(status, SPEC_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+          "r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// K-major operand in 128-byte swizzled atoms (rows of 128 bytes, 8-row
+// groups 1024 bytes apart): start address, SBO = 1024, descriptor version 1,
+// layout SWIZZLE_128B.
+__device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1 << 16;             // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;   // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;             // descriptor version
+  d |= (uint64_t)2 << 61;             // SWIZZLE_128B
+  return d;
+}
+// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, both
+// K-major, N and M.
+__host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int k = 0; k < 32; ++k) v[k] = __uint_as_float(r[k]);
+}
+
+// ---------------------------------------------------------------------------
+// Level-1 keys as in draft.cu (log2 domain, compared as differences)
+// ---------------------------------------------------------------------------
+struct MkKey {
+  float L, M;
+  int32_t idx;
+};
+__device__ __forceinline__ bool mk_better(const MkKey& a, const MkKey& b, float c2) {
+  if (a.idx == INT_MAX) return false;
+  if (b.idx == INT_MAX) return true;
+  const float lhs = a.L - b.L, rhs = c2 * (a.M - b.M);
+  return lhs < rhs || (lhs == rhs && a.idx < b.idx);
+}
+__device__ __forceinline__ SoftState mk_merge(SoftState a, SoftState b, float c2) {
+  if (b.m > a.m) {
+    const SoftState t = a;
+    a = b;
+    b = t;
+  }
+  if (b.m == -INFINITY) return a;
+  a.s = a.s + b.s * ex2_approx(b.m * c2 - a.m * c2);
+  return a;
+}
+__device__ __forceinline__ float mk_lg2(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// ---------------------------------------------------------------------------
+// The bias and level-1 pass of one position
+// ---------------------------------------------------------------------------
+template <bool kGreedy>
+__global__ void __launch_bounds__(kMkThreads, 1)
+    markov_bias_kernel(const __grid_constant__ CUtensorMap tmE, const __grid_constant__ CUtensorMap tmW,
+                       const MarkovLaunch p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int nk = p.r / kMkAtomK;
+  uint8_t* sA = smem;                          // nk atoms
+  uint8_t* sB = smem + nk * kMkAtomBytes;      // 2 stages of nk atoms
+  __shared__ uint64_t bar_a, bar_full[2], bar_mma[2], bar_free[2];
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int abort_flag;
+  volatile int& abort_sh = abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nb = (p.V + kRaceBlock - 1) / kRaceBlock;
+  const int my_blocks = nb > (int)blockIdx.x ? (nb - 1 - (int)blockIdx.x) / p.G + 1 : 0;
+  const int T = 2 * my_blocks;                 // tiles: two halves per race block
+  // epilogue warps with at least one request row
+  const int n_epi = (p.B + 31) / 32;
+  const bool epi = warp >= 2;
+  const int q = warp & 3;                      // TMEM lane quarter of this warp
+  const bool epi_active = epi && 32 * q < p.B;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bar_a, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_mma[s], 1);
+      mbar_init(&bar_free[s], (uint32_t)n_epi);
+    }
+    abort_sh = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base_sh)),
+                 "r"(kMkTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_sh;
+
+  if (warp == 0) {
+    // ---- TMA producer ----
+    if (lane == 0 && T > 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmE)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
+      mbar_expect_tx(&bar_a, (uint32_t)(nk * kMkAtomBytes));
+      for (int a = 0; a < nk; ++a) tma_load_2d(sA + a * kMkAtomBytes, &tmE, a * kMkAtomK, 0, &bar_a);
+      for (int t = 0; t < T; ++t) {
+        const int s = t & 1, u = t >> 1;
+        if (u > 0 && !mbar_wait(&bar_mma[s], (uint32_t)((u - 1) & 1), p.status)) {
+          abort_sh = 1;
+          break;
+        }
+        if (abort_sh) break;
+        const int v0 = ((int)blockIdx.x + (t >> 1) * p.G) * kRaceBlock + (t & 1) * kMkTile;
+        mbar_expect_tx(&bar_full[s], (uint32_t)(nk * kMkAtomBytes));
+        for (int a = 0; a < nk; ++a)
+          tma_load_2d(sB + (s * nk + a) * kMkAtomBytes, &tmW, a * kMkAtomK, v0, &bar_full[s]);
+      }
+    }
+  } else if (warp == 1) {
+    // ---- MMA issuer ----
+    int issued = 0;
+    if (lane == 0 && T > 0) {
+      constexpr uint32_t idesc = umma_idesc_bf16(kMkRows, kMkTile);
+      if (!mbar_wait(&bar_a, 0u, p.status)) abort_sh = 1;
+      for (int t = 0; t < T && !abort_sh; ++t) {
+        const int s = t & 1, u = t >> 1;
+        if (u > 0 && !mbar_wait(&bar_free[s], (uint32_t)((u - 1) & 1), p.status)) {
+          abort_sh = 1;
+          break;
+        }
+        if (!mbar_wait(&bar_full[s], (uint32_t)(u & 1), p.status)) {
+          abort_sh = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(s * kMkTile);
+        for (int kk = 0; kk < p.r / 16; ++kk) {
+          const uint32_t koff = (uint32_t)((kk >> 2) * kMkAtomBytes + (kk & 3) * 32);
+          const uint64_t da = umma_desc_sw128(smem_u32(sA) + koff);
+          const uint64_t db = umma_desc_sw128(smem_u32(sB + s * nk * kMkAtomBytes) + koff);
+          umma_bf16(d, da, db, idesc, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&bar_mma[s]);
+        issued = t + 1;
+      }
+      // what was issued completes before the TMEM is freed
+      if (issued > 0) mbar_wait(&bar_mma[(issued - 1) & 1], (uint32_t)(((issued - 1) >> 1) & 1), p.status);
+    }
+    __syncwarp();
+  } else if (epi_active) {
+    // ---- epilogue: one request row per thread ----
+    const int row = 32 * q + lane;
+    const bool valid = row < p.B;
+    const size_t urow = ((size_t)(valid ? row : 0) * p.K + p.step) * (size_t)p.V;
+    const long long pos = valid ? __ldg(reinterpret_cast<const long long*>(p.pos_base) + row) : 0;
+    const uint32_t position = (uint32_t)(pos + p.step + 1);
+    const uint64_t req = valid ? __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + row) : 0;
+    const uint64_t seed = valid ? __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + row) : 0;
+    SoftState st{-INFINITY, 0.0f};
+    MkKey best{INFINITY, 0.0f, INT_MAX};
+    ArgState g{-INFINITY, INT_MAX};
+    int32_t flags = 0;
+    SoftState half{-INFINITY, 0.0f};  // the current race block's two halves
+    bool aborted = false;
+    for (int t = 0; t < T; ++t) {
+      const int s = t & 1, u = t >> 1;
+      const int b = (int)blockIdx.x + (t >> 1) * p.G;
+      const int v0 = b * kRaceBlock + (t & 1) * kMkTile;
+      // this tile's 128 entries of U (bf16), fetched before the accumulator wait
+      uint4 uw[16];
+#pragma unroll
+      for (int h = 0; h < 16; ++h) {
+        const int v = v0 + 8 * h;
+        if (valid && p.u_vec && v + 8 <= p.V) {
+          uw[h] = ldg_stream(p.U + urow + v);
+        } else {
+          uint32_t e[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            e[j] = (valid && v + j < p.V) ? (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p.U) + urow + v + j)
+                                          : 0xFF80u;  // -inf past V
+          uw[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
+        }
+      }
+      const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(&bar_mma[s], (uint32_t)(u & 1), p.status));
+      if (!ok) {
+        aborted = true;
+        break;
+      }
+      tc_fence_after();
+      // the tile's 4 chunks of 32 columns, each merged online: its max (and
+      // first argmax) and its sum relative to that max
+      SoftState tile{-INFINITY, 0.0f};
+#pragma unroll
+      for (int ch = 0; ch < kMkTile / 32; ++ch) {
+        float l[32];
+        tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(s * kMkTile + 32 * ch), l);
+        float cmax = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const uint4& w4 = uw[(32 * ch + k) >> 3];
+          const int e = k & 7;
+          const uint32_t word = e < 2 ? w4.x : e < 4 ? w4.y : e < 6 ? w4.z : w4.w;
+          l[k] += (e & 1) ? bf16_hi(word) : bf16_lo(word);  // -inf past V (U reads -inf there, the bias is 0)
+          cmax = fmaxf(cmax, l[k]);
+        }
+        if (!valid) continue;
+        if (cmax == INFINITY) flags |= 1;
+        if (kGreedy && cmax > -INFINITY && (g.idx == INT_MAX || cmax > g.v)) {
+          int first = INT_MAX;
+#pragma unroll
+          for (int k = 31; k >= 0; --k)
+            if (l[k] == cmax) first = v0 + 32 * ch + k;
+          g = ArgState{cmax, first};
+        }
+        if (cmax > -INFINITY && cmax < INFINITY) {
+          const float M2 = cmax * p.c2;
+          float cs = 0.0f;
+#pragma unroll
+          for (int k = 0; k < 32; ++k) cs += ex2_approx(__fmaf_rn(l[k], p.c2, -M2));
+          if (cs != cs) flags |= 1;  // a NaN entry
+          else tile = mk_merge(tile, SoftState{cmax, cs}, p.c2);
+        } else if (cmax != cmax) {
+          flags |= 1;
+        }
+      }
+      // the accumulator is read: the MMA may overwrite it
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar_free[s]);
+      if (!valid) continue;
+      half = mk_merge(half, tile, p.c2);
+      if ((t & 1) == 1 || t == T - 1) {
+        // the race block is complete
+        st = mk_merge(st, half, p.c2);
+        if (!kGreedy && half.m > -INFINITY && half.s > 0.0f && half.s == half.s) {
+          const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)(b >> 2)), (uint32_t)seed,
+                                  (uint32_t)(seed >> 32));
+          const uint32_t word = (b & 3) == 0 ? rq.x : (b & 3) == 1 ? rq.y : (b & 3) == 2 ? rq.z : rq.w;
+          const float E = -log1pf(-((float)race_m(word) * 0x1p-24f));
+          const MkKey cand{mk_lg2(E) - mk_lg2(half.s), half.m, b};
+          if (mk_better(cand, best, p.c2)) best = cand;
+        }
+        half = SoftState{-INFINITY, 0.0f};
+      }
+    }
+    if (valid && !aborted) {
+      MkPartial o{};
+      o.m = st.m;
+      o.s = st.s;
+      o.L = kGreedy ? g.v : best.L;
+      o.idx = kGreedy ? g.idx : best.idx;
+      o.M = best.M;
+      o.flags = flags;
+      p.part[(size_t)row * p.G + blockIdx.x] = o;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kMkTmemCols) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// The draw of one position: merge, level 2, outputs, next E
+// ---------------------------------------------------------------------------
+template <bool kGreedy>
+__global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovLaunch p) {
+  __shared__ __align__(16) __nv_bfloat16 sh_e[kMkMaxR];
+  __shared__ float sh_l[kPickThreads];
+  __shared__ KeyState sh_red[kPickThreads / 32];
+  __shared__ float sh_m, sh_S;
+  __shared__ int sh_idx, sh_bad;
+  const int i = blockIdx.x;
+  const int lane = threadIdx.x & 31;
+  pdl_wait_prerequisites();
+  for (int j = threadIdx.x; j < p.r; j += kPickThreads) sh_e[j] = p.E[(size_t)i * p.r + j];
+  if (threadIdx.x < 32) {
+    SoftState st{-INFINITY, 0.0f};
+    MkKey best{INFINITY, 0.0f, INT_MAX};
+    ArgState g{-INFINITY, INT_MAX};
+    int32_t f = 0;
+    for (int c = lane; c < p.G; c += 32) {
+      const MkPartial o = p.part[(size_t)i * p.G + c];
+      st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
+      f |= o.flags;
+      if (kGreedy) {
+        const ArgState a{o.L, o.idx};
+        if (arg_better(a, g)) g = a;
+      } else {
+        const MkKey k{o.L, o.M, o.idx};
+        if (mk_better(k, best, p.c2)) best = k;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      st = soft_merge(st, SoftState{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)},
+                      p.c2);
+      const MkKey ok{__shfl_xor_sync(0xFFFFFFFFu, best.L, o), __shfl_xor_sync(0xFFFFFFFFu, best.M, o),
+                     __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
+      if (mk_better(ok, best, p.c2)) best = ok;
+      const ArgState og{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
+      if (arg_better(og, g)) g = og;
+    }
+    f = (int32_t)__reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
+    if (lane == 0) {
+      sh_m = st.m;
+      sh_S = st.s;
+      sh_idx = kGreedy ? g.idx : best.idx;
+      sh_bad = (f || p.req_bad[i] || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
+                   ? 1 : 0;
+    }
+  }
+  __syncthreads();
+  const bool bad = sh_bad != 0;
+  const float M2 = sh_m * p.c2;
+  int z = -1;
+  float lz = sh_m;
+  if (!bad) {
+    if (kGreedy) {
+      z = sh_idx;
+    } else {
+      // level 2: the winning block's logits recomputed (U + E . W2^T row)
+      const int b = sh_idx;
+      const int v = b * kRaceBlock + (int)threadIdx.x;
+      KeyState e{INFINITY, INT_MAX};
+      float l = -INFINITY;
+      if (v < p.V) {
+        const __nv_bfloat16* wrow = p.W2T + (size_t)v * p.r;
+        float dot = 0.0f;
+        for (int j = 0; j < p.r; j += 8) {
+          const uint4 w8 = __ldg(reinterpret_cast<const uint4*>(wrow + j));
+          const uint4 e8 = *reinterpret_cast<const uint4*>(sh_e + j);
+          const uint32_t ww[4] = {w8.x, w8.y, w8.z, w8.w}, ee[4] = {e8.x, e8.y, e8.z, e8.w};
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            dot = fmaf(bf16_lo(ee[h]), bf16_lo(ww[h]), dot);
+            dot = fmaf(bf16_hi(ee[h]), bf16_hi(ww[h]), dot);
+          }
+        }
+        l = load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) + dot;
+        const float w = ex2_approx(__fmaf_rn(l, p.c2, -M2));
+        const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
+        const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
+        const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+        const uint4 rw = philox(draw_counter((uint32_t)(pos + p.step + 1), req, SPEC_PURPOSE_DRAFT_IN_BLOCK,
+                                             (uint32_t)(v >> 2)),
+                                (uint32_t)seed, (uint32_t)(seed >> 32));
+        const uint32_t word = (v & 3) == 0 ? rw.x : (v & 3) == 1 ? rw.y : (v & 3) == 2 ? rw.z : rw.w;
+        if (w > 0.0f) e = KeyState{race_key(race_m(word), w), v};
+      }
+      sh_l[threadIdx.x] = l;
+      e = cta_min_key(e, sh_red);
+      if (threadIdx.x == 0) sh_idx = e.idx == INT_MAX ? -1 : e.idx;
+      __syncthreads();
+      z = sh_idx;
+      if (z >= 0) lz = sh_l[z - b * kRaceBlock];
+    }
+  }
+  // the next position's operand row: W1 at this draft
+  if (p.step + 1 < p.K)
+    for (int j = threadIdx.x; j < p.r; j += kPickThreads)
+      p.E[(size_t)i * p.r + j] = p.W1[(size_t)(bad || z < 0 ? 0 : z) * p.r + j];
+  if (threadIdx.x != 0) return;
+  const size_t o = (size_t)i * p.K + p.step;
+  if (bad || z < 0) {
+    p.req_bad[i] = 1u;
+    p.drafts[o] = -1;
+    p.conf[o] = 0.0f;
+    if (p.row_stats) reinterpret_cast<float2*>(p.row_stats)[o] = make_float2(0.0f, 0.0f);
+  } else {
+    p.drafts[o] = z;
+    p.conf[o] = exp2f(fmaf(lz, p.c2, -M2)) / sh_S;
+    if (p.row_stats) {
+      const float resid = fmaf(sh_m, p.c2, -M2);
+      reinterpret_cast<float2*>(p.row_stats)[o] = make_float2(sh_m * p.inv_t, (log2f(sh_S) - resid) * 0.69314718055994531f);
+    }
+  }
+  if (p.step + 1 < p.K) return;
+  // ---- the last position: a bad request's outputs, the scores ----
+  const bool req_bad = p.req_bad[i] != 0u;
+  if (req_bad) {
+    p.req_bad[i] = 0u;  // leave the workspace zeroed for the next call
+    report(p.status, SPEC_ERR_BAD_INPUT);
+    for (int k = 0; k < p.K; ++k) {
+      p.drafts[(size_t)i * p.K + k] = -1;
+      p.conf[(size_t)i * p.K + k] = 0.0f;
+      if (p.row_stats) reinterpret_cast<float2*>(p.row_stats)[(size_t)i * p.K + k] = make_float2(0.0f, 0.0f);
+    }
+  }
+  if (p.scores) {
+    float* sc = p.scores + (size_t)i * (p.K + 1);
+    float run = 1.0f;
+    sc[0] = run;
+    for (int k = 0; k < p.K; ++k) {
+      run = req_bad ? 0.0f : __fmul_rn(run, p.conf[(size_t)i * p.K + k]);
+      sc[k + 1] = run;
+    }
+  }
+}
+
+// The first position's operand: W1 at the last committed tokens; rows past B
+// zero (the padding rows of the MMA).  One CTA per row of E.
+__global__ void __launch_bounds__(128) markov_begin_kernel(const MarkovLaunch p) {
+  const int i = blockIdx.x;
+  pdl_wait_prerequisites();
+  int x = 0;
+  bool bad = true;
+  if (i < p.B) {
+    x = __ldg(p.x0 + i);
+    const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
+    bad = x < 0 || x >= p.V || pos < 0 || pos + p.K > 0xFFFFFFFFLL;
+    if (threadIdx.x == 0) p.req_bad[i] = bad ? 1u : 0u;
+  }
+  for (int j = threadIdx.x; j < p.r; j += blockDim.x)
+    p.E[(size_t)i * p.r + j] = (i < p.B && !bad) ? p.W1[(size_t)x * p.r + j] : __float2bfloat16(0.0f);
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// A [rows, r] bf16 matrix in boxes of 64 (K) x 128 (rows), 128-byte swizzle.
+static bool make_map(CUtensorMap* map, const void* base, int r, long long rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)r, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)r * 2};
+  cuuint32_t box[2] = {(cuuint32_t)kMkAtomK, 128u};
+  cuuint32_t estr[2] = {1u, 1u};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct MarkovGeometry {
+  int G;
+  size_t e_off, part_off, bad_off, bytes;
+};
+
+static MarkovGeometry markov_geometry(int B, int V, int r, int sms) {
+  MarkovGeometry g{};
+  const int nb = (V + kRaceBlock - 1) / kRaceBlock;
+  g.G = std::max(1, std::min(sms, nb));
+  g.e_off = 0;
+  g.part_off = ((size_t)kMkRows * r * 2 + 255) / 256 * 256;
+  g.bad_off = g.part_off + ((size_t)sizeof(MkPartial) * B * g.G + 255) / 256 * 256;
+  g.bytes = g.bad_off + ((size_t)4 * B + 255) / 256 * 256;
+  return g;
+}
+
+static int device_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 1;
+  return sms;
+}
+
+static bool markov_shape_ok(int B, int K, int V, int r) {
+  return B >= 1 && B <= kMkRows && K >= 1 && K <= SPEC_MAX_DRAFTS && V >= 1 && V < SPEC_MAX_VOCAB && r >= kMkAtomK &&
+         r <= kMkMaxR && r % kMkAtomK == 0;
+}
+
+}  // namespace spec
+
+extern "C" size_t spec_markov_workspace(int B, int K, int V, int r) {
+  if (!spec::markov_shape_ok(B, K, V, r)) return 0;
+  // sized for up to 1024 SMs, so that the size does not depend on the device
+  return spec::markov_geometry(B, V, r, 1024).bytes;
+}
+
+extern "C" int spec_markov_draft(const void* U, int u_dtype, const void* W1, const void* W2T, int r,
+                                 const int32_t* x0, int B, int K, int V, float tau, const uint64_t* seeds,
+                                 const uint64_t* request_ids, const int64_t* pos_base, int32_t* drafts_out,
+                                 float* conf_out, float* scores_out, float* row_stats_out, int32_t* status,
+                                 void* ws, size_t ws_bytes, cudaStream_t stream) {
+  using namespace spec;
+  if (!markov_shape_ok(B, K, V, r) || u_dtype != SPEC_BF16 || !(tau >= 0.0f) || isinf(tau))
+    return SPEC_ERR_INVALID_ARG;
+  if (!U || !W1 || !W2T || !x0 || !seeds || !request_ids || !pos_base || !drafts_out || !conf_out)
+    return SPEC_ERR_INVALID_ARG;
+  if (((reinterpret_cast<uintptr_t>(W1) | reinterpret_cast<uintptr_t>(W2T)) & 15u) != 0 ||
+      (row_stats_out && (reinterpret_cast<uintptr_t>(row_stats_out) & 7u) != 0))
+    return SPEC_ERR_INVALID_ARG;
+  const int sms = device_sms();
+  const MarkovGeometry g = markov_geometry(B, V, r, std::min(sms, 1024));
+  if (!ws || ws_bytes < g.bytes || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return SPEC_ERR_WORKSPACE;
+  MarkovLaunch p{};
+  p.U = static_cast<const __nv_bfloat16*>(U);
+  p.W1 = static_cast<const __nv_bfloat16*>(W1);
+  p.W2T = static_cast<const __nv_bfloat16*>(W2T);
+  p.r = r;
+  p.B = B;
+  p.K = K;
+  p.V = V;
+  p.tau = tau;
+  const double tc = tau > 0.0f ? (double)tau : 1.0;
+  p.c2 = (float)(1.4426950408889634 / tc);
+  p.inv_t = (float)(1.0 / tc);
+  p.seeds = seeds;
+  p.request_ids = request_ids;
+  p.pos_base = pos_base;
+  p.x0 = x0;
+  char* base = static_cast<char*>(ws);
+  p.E = reinterpret_cast<__nv_bfloat16*>(base + g.e_off);
+  p.part = reinterpret_cast<MkPartial*>(base + g.part_off);
+  p.G = g.G;
+  p.req_bad = reinterpret_cast<uint32_t*>(base + g.bad_off);
+  p.drafts = drafts_out;
+  p.conf = conf_out;
+  p.scores = scores_out;
+  p.row_stats = row_stats_out;
+  p.status = status;
+  p.u_vec = (reinterpret_cast<uintptr_t>(U) & 15u) == 0 && V % 8 == 0;
+  CUtensorMap tmE, tmW;
+  if (!make_map(&tmE, p.E, r, kMkRows) || !make_map(&tmW, W2T, r, V)) return SPEC_ERR_CUDA;
+  const int nk = r / kMkAtomK;
+  const size_t smem = 1024 + (size_t)3 * nk * kMkAtomBytes;
+  const bool greedy = tau == 0.0f;
+  auto bias = greedy ? markov_bias_kernel<true> : markov_bias_kernel<false>;
+  auto pick = greedy ? markov_pick_kernel<true> : markov_pick_kernel<false>;
+  if (cudaFuncSetAttribute(bias, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return SPEC_ERR_CUDA;
+  cudaError_t err = launch_after_previous(markov_begin_kernel, dim3(kMkRows), dim3(128), 0, stream, p);
+  for (int k = 0; k < K && err == cudaSuccess; ++k) {
+    p.step = k;
+    // the bias kernel holds the SM's TMEM: launched after its predecessor completes
+    bias<<<g.G, kMkThreads, smem, stream>>>(tmE, tmW, p);
+    err = cudaGetLastError();
+    if (err == cudaSuccess) err = launch_after_previous(pick, dim3(B), dim3(kPickThreads), 0, stream, p);
+  }
+  if (err != cudaSuccess || cudaGetLastError() != cudaSuccess) return SPEC_ERR_CUDA;
+  return SPEC_OK;
+}
