@@ -13,12 +13,14 @@
 //                       once and then tiles of W2^T (128 vocabulary rows x r,
 //                       128-byte swizzle), double-buffered.  Warp 1 issues
 //                       tcgen05.mma (M = 128, N = 128, K = 16, bf16 -> fp32)
-//                       into two TMEM accumulators.  The epilogue warps read
-//                       the accumulator rows (tcgen05.ld, one request per
-//                       thread), add U_k, and per race block of 256 entries
+//                       into four TMEM accumulators.  Eight epilogue warps (two
+//                       per TMEM lane quarter, alternate race blocks) read the
+//                       accumulator rows (tcgen05.ld, one request per thread),
+//                       add U_k, and per race block of 256 entries
 //                       form the block's max and sum, its level-1 race key
 //                       (or its argmax at tau = 0) and the row's softmax
-//                       statistics.  Each CTA writes one partial per request.
+//                       statistics.  Each epilogue half of a CTA writes one
+//                       partial per request.
 //   markov_pick_kernel  one CTA per request: merges the partials, recomputes
 //                       the winning block's 256 logits and draws inside it
 //                       (level 2), writes the draft, its confidence and the
@@ -41,9 +43,11 @@ constexpr int kMkRows = 128;        // MMA M: request rows (rows >= B are zero)
 constexpr int kMkTile = 128;        // MMA N: vocabulary rows of W2^T per tile
 constexpr int kMkAtomK = 64;        // bf16 along K per 128-byte swizzle atom
 constexpr int kMkAtomBytes = 128 * 128;  // one atom of 128 rows x 128 bytes
-constexpr int kMkThreads = 192;     // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kMkEpiWarps = 8;      // two per TMEM lane quarter, taking alternate race blocks
+constexpr int kMkThreads = 32 * (2 + kMkEpiWarps);  // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr int kMkMaxR = 256;
-constexpr int kMkTmemCols = 256;    // two accumulators of kMkTile fp32 columns
+constexpr int kMkSlots = 4;         // accumulators: (smem stage) x (epilogue half)
+constexpr int kMkTmemCols = kMkSlots * kMkTile;  // 512 fp32 columns
 constexpr int kPickThreads = 256;
 
 struct alignas(16) MkPartial {
@@ -66,7 +70,7 @@ struct MarkovLaunch {
   const int64_t* pos_base;
   const int32_t* x0;
   __nv_bfloat16* E;  // [128, r]: W1 at the previous drafts
-  MkPartial* part;   // [B][G]
+  MkPartial* part;   // [B][2G]: one per epilogue half of each bias CTA
   int G;
   uint32_t* req_bad;  // [B]
   int32_t* drafts;
@@ -220,7 +224,11 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int nk = p.r / kMkAtomK;
   uint8_t* sA = smem;                          // nk atoms
   uint8_t* sB = smem + nk * kMkAtomBytes;      // 2 stages of nk atoms
-  __shared__ uint64_t bar_a, bar_full[2], bar_mma[2], bar_free[2];
+  // Tile t uses smem stage t & 1 and accumulator slot t & 3 (stage + 2 x the
+  // epilogue half of its race block), so that every waiter of a barrier sees
+  // its phases one after another (a parity wait two phases behind would
+  // alias).
+  __shared__ uint64_t bar_a, bar_full[2], bar_mma[kMkSlots], bar_free[kMkSlots];
   __shared__ uint32_t tmem_base_sh;
   __shared__ int abort_flag;
   volatile int& abort_sh = abort_flag;
@@ -232,14 +240,17 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int n_epi = (p.B + 31) / 32;
   const bool epi = warp >= 2;
   const int q = warp & 3;                      // TMEM lane quarter of this warp
+  const int eh = (warp - 2) >> 2;              // epilogue half: the race blocks j with j % 2 == eh
   const bool epi_active = epi && 32 * q < p.B;
 
+  // E and the partials are read and written by the kernels around this one
+  pdl_wait_prerequisites();
   if (threadIdx.x == 0) {
     mbar_init(&bar_a, 1);
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&bar_full[s], 1);
-      mbar_init(&bar_mma[s], 1);
-      mbar_init(&bar_free[s], (uint32_t)n_epi);
+    for (int s = 0; s < 2; ++s) mbar_init(&bar_full[s], 1);
+    for (int k = 0; k < kMkSlots; ++k) {
+      mbar_init(&bar_mma[k], 1);
+      mbar_init(&bar_free[k], (uint32_t)n_epi);
     }
     abort_sh = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -263,8 +274,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       mbar_expect_tx(&bar_a, (uint32_t)(nk * kMkAtomBytes));
       for (int a = 0; a < nk; ++a) tma_load_2d(sA + a * kMkAtomBytes, &tmE, a * kMkAtomK, 0, &bar_a);
       for (int t = 0; t < T; ++t) {
-        const int s = t & 1, u = t >> 1;
-        if (u > 0 && !mbar_wait(&bar_mma[s], (uint32_t)((u - 1) & 1), p.status)) {
+        const int s = t & 1;
+        // the stage's previous tile (t - 2) has been consumed by its MMA
+        if (t >= 2 && !mbar_wait(&bar_mma[(t - 2) & 3], (uint32_t)(((t - 2) >> 2) & 1), p.status)) {
           abort_sh = 1;
           break;
         }
@@ -282,8 +294,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       constexpr uint32_t idesc = umma_idesc_bf16(kMkRows, kMkTile);
       if (!mbar_wait(&bar_a, 0u, p.status)) abort_sh = 1;
       for (int t = 0; t < T && !abort_sh; ++t) {
-        const int s = t & 1, u = t >> 1;
-        if (u > 0 && !mbar_wait(&bar_free[s], (uint32_t)((u - 1) & 1), p.status)) {
+        const int s = t & 1, u = t >> 1, slot = t & 3;
+        // the slot's previous tile (t - 4) has been read by the epilogue
+        if (t >= kMkSlots && !mbar_wait(&bar_free[slot], (uint32_t)(((t >> 2) - 1) & 1), p.status)) {
           abort_sh = 1;
           break;
         }
@@ -292,18 +305,18 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(s * kMkTile);
+        const uint32_t d = tmem + (uint32_t)(slot * kMkTile);
         for (int kk = 0; kk < p.r / 16; ++kk) {
           const uint32_t koff = (uint32_t)((kk >> 2) * kMkAtomBytes + (kk & 3) * 32);
           const uint64_t da = umma_desc_sw128(smem_u32(sA) + koff);
           const uint64_t db = umma_desc_sw128(smem_u32(sB + s * nk * kMkAtomBytes) + koff);
           umma_bf16(d, da, db, idesc, kk > 0 ? 1u : 0u);
         }
-        umma_commit(&bar_mma[s]);
+        umma_commit(&bar_mma[slot]);
         issued = t + 1;
       }
       // what was issued completes before the TMEM is freed
-      if (issued > 0) mbar_wait(&bar_mma[(issued - 1) & 1], (uint32_t)(((issued - 1) >> 1) & 1), p.status);
+      if (issued > 0) mbar_wait(&bar_mma[(issued - 1) & 3], (uint32_t)(((issued - 1) >> 2) & 1), p.status);
     }
     __syncwarp();
   } else if (epi_active) {
@@ -321,27 +334,32 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     int32_t flags = 0;
     SoftState half{-INFINITY, 0.0f};  // the current race block's two halves
     bool aborted = false;
-    for (int t = 0; t < T; ++t) {
-      const int s = t & 1, u = t >> 1;
-      const int b = (int)blockIdx.x + (t >> 1) * p.G;
-      const int v0 = b * kRaceBlock + (t & 1) * kMkTile;
-      // this tile's 128 entries of U (bf16), fetched before the accumulator wait
-      uint4 uw[16];
+    // a tile's 128 entries of U (bf16), loaded one tile ahead of their use
+    auto load_u = [&](int t, uint4 (&w)[16]) {
+      const int v0 = ((int)blockIdx.x + (t >> 1) * p.G) * kRaceBlock + (t & 1) * kMkTile;
 #pragma unroll
       for (int h = 0; h < 16; ++h) {
         const int v = v0 + 8 * h;
         if (valid && p.u_vec && v + 8 <= p.V) {
-          uw[h] = ldg_stream(p.U + urow + v);
+          w[h] = ldg_stream(p.U + urow + v);
         } else {
           uint32_t e[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j)
             e[j] = (valid && v + j < p.V) ? (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p.U) + urow + v + j)
                                           : 0xFF80u;  // -inf past V
-          uw[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
+          w[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
         }
       }
-      const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(&bar_mma[s], (uint32_t)(u & 1), p.status));
+    };
+    uint4 uw[16];
+    for (int t = 0; t < T; ++t) {
+      if (((t >> 1) & 1) != eh) continue;  // the other half's race block
+      const int slot = t & 3;
+      const int b = (int)blockIdx.x + (t >> 1) * p.G;
+      const int v0 = b * kRaceBlock + (t & 1) * kMkTile;
+      load_u(t, uw);  // issued before the accumulator wait
+      const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(&bar_mma[slot], (uint32_t)((t >> 2) & 1), p.status));
       if (!ok) {
         aborted = true;
         break;
@@ -353,7 +371,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 #pragma unroll
       for (int ch = 0; ch < kMkTile / 32; ++ch) {
         float l[32];
-        tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(s * kMkTile + 32 * ch), l);
+        tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(slot * kMkTile + 32 * ch), l);
         float cmax = -INFINITY;
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
@@ -386,7 +404,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       // the accumulator is read: the MMA may overwrite it
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bar_free[s]);
+      if (lane == 0) mbar_arrive(&bar_free[slot]);
       if (!valid) continue;
       half = mk_merge(half, tile, p.c2);
       if ((t & 1) == 1 || t == T - 1) {
@@ -411,7 +429,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       o.idx = kGreedy ? g.idx : best.idx;
       o.M = best.M;
       o.flags = flags;
-      p.part[(size_t)row * p.G + blockIdx.x] = o;
+      p.part[(size_t)row * 2 * p.G + 2 * blockIdx.x + eh] = o;
     }
   }
   tc_fence_before();
@@ -441,8 +459,8 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    for (int c = lane; c < p.G; c += 32) {
-      const MkPartial o = p.part[(size_t)i * p.G + c];
+    for (int c = lane; c < 2 * p.G; c += 32) {
+      const MkPartial o = p.part[(size_t)i * 2 * p.G + c];
       st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
       f |= o.flags;
       if (kGreedy) {
@@ -481,25 +499,54 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
     if (kGreedy) {
       z = sh_idx;
     } else {
-      // level 2: the winning block's logits recomputed (U + E . W2^T row)
+      // level 2: the winning block's logits recomputed (U + E . W2^T row).
+      // Warp w takes entries 32w..32w+31 of the block; lane l multiplies the
+      // r-slice 8l..8l+7 of each (one coalesced 16-byte load per entry, all
+      // issued at once), and a transposed butterfly leaves entry 32w + l's
+      // dot product in lane l.
       const int b = sh_idx;
-      const int v = b * kRaceBlock + (int)threadIdx.x;
+      const int w_id = threadIdx.x >> 5;
+      const int v_base = b * kRaceBlock + 32 * w_id;
+      float part[32];
+      {
+        const bool has = 8 * lane < p.r;
+        uint4 e8 = make_uint4(0u, 0u, 0u, 0u);
+        if (has) e8 = *reinterpret_cast<const uint4*>(sh_e + 8 * lane);
+        const uint32_t ee[4] = {e8.x, e8.y, e8.z, e8.w};
+        uint4 w8[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          w8[j] = (has && v_base + j < p.V) ? __ldg(reinterpret_cast<const uint4*>(p.W2T + (size_t)(v_base + j) * p.r) + lane)
+                                            : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const uint32_t ww[4] = {w8[j].x, w8[j].y, w8[j].z, w8[j].w};
+          float acc = 0.0f;
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            acc = fmaf(bf16_lo(ee[h]), bf16_lo(ww[h]), acc);
+            acc = fmaf(bf16_hi(ee[h]), bf16_hi(ww[h]), acc);
+          }
+          part[j] = acc;
+        }
+      }
+      // transposed butterfly: 16 + 8 + 4 + 2 + 1 exchanges
+#pragma unroll
+      for (int n = 32, o = 16; n > 1; n >>= 1, o >>= 1) {
+        const bool hi = (lane & o) != 0;
+#pragma unroll
+        for (int j = 0; j < n / 2; ++j) {
+          const float send = hi ? part[j] : part[j + n / 2];
+          const float keep = hi ? part[j + n / 2] : part[j];
+          part[j] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
+        }
+      }
+      // lane l now holds entry 32w + l (the halving kept the block of l's bits)
+      const int v = v_base + lane;
       KeyState e{INFINITY, INT_MAX};
       float l = -INFINITY;
       if (v < p.V) {
-        const __nv_bfloat16* wrow = p.W2T + (size_t)v * p.r;
-        float dot = 0.0f;
-        for (int j = 0; j < p.r; j += 8) {
-          const uint4 w8 = __ldg(reinterpret_cast<const uint4*>(wrow + j));
-          const uint4 e8 = *reinterpret_cast<const uint4*>(sh_e + j);
-          const uint32_t ww[4] = {w8.x, w8.y, w8.z, w8.w}, ee[4] = {e8.x, e8.y, e8.z, e8.w};
-#pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            dot = fmaf(bf16_lo(ee[h]), bf16_lo(ww[h]), dot);
-            dot = fmaf(bf16_hi(ee[h]), bf16_hi(ww[h]), dot);
-          }
-        }
-        l = load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) + dot;
+        l = load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) + part[0];
         const float w = ex2_approx(__fmaf_rn(l, p.c2, -M2));
         const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
         const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
@@ -510,7 +557,7 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
         const uint32_t word = (v & 3) == 0 ? rw.x : (v & 3) == 1 ? rw.y : (v & 3) == 2 ? rw.z : rw.w;
         if (w > 0.0f) e = KeyState{race_key(race_m(word), w), v};
       }
-      sh_l[threadIdx.x] = l;
+      sh_l[v - b * kRaceBlock] = l;
       e = cta_min_key(e, sh_red);
       if (threadIdx.x == 0) sh_idx = e.idx == INT_MAX ? -1 : e.idx;
       __syncthreads();
@@ -617,7 +664,7 @@ static MarkovGeometry markov_geometry(int B, int V, int r, int sms) {
   g.G = std::max(1, std::min(sms, nb));
   g.e_off = 0;
   g.part_off = ((size_t)kMkRows * r * 2 + 255) / 256 * 256;
-  g.bad_off = g.part_off + ((size_t)sizeof(MkPartial) * B * g.G + 255) / 256 * 256;
+  g.bad_off = g.part_off + ((size_t)sizeof(MkPartial) * B * 2 * g.G + 255) / 256 * 256;
   g.bytes = g.bad_off + ((size_t)4 * B + 255) / 256 * 256;
   return g;
 }
@@ -697,9 +744,9 @@ extern "C" int spec_markov_draft(const void* U, int u_dtype, const void* W1, con
   cudaError_t err = launch_after_previous(markov_begin_kernel, dim3(kMkRows), dim3(128), 0, stream, p);
   for (int k = 0; k < K && err == cudaSuccess; ++k) {
     p.step = k;
-    // the bias kernel holds the SM's TMEM: launched after its predecessor completes
-    bias<<<g.G, kMkThreads, smem, stream>>>(tmE, tmW, p);
-    err = cudaGetLastError();
+    // one CTA per SM (shared memory): a CTA launched early waits in
+    // griddepcontrol.wait for the previous position's pick kernel
+    err = launch_after_previous(bias, dim3(g.G), dim3(kMkThreads), smem, stream, tmE, tmW, p);
     if (err == cudaSuccess) err = launch_after_previous(pick, dim3(B), dim3(kPickThreads), 0, stream, p);
   }
   if (err != cudaSuccess || cudaGetLastError() != cudaSuccess) return SPEC_ERR_CUDA;
