@@ -454,12 +454,14 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
   const int lane = threadIdx.x & 31;
   pdl_wait_prerequisites();
   for (int j = threadIdx.x; j < p.r; j += kPickThreads) sh_e[j] = p.E[(size_t)i * p.r + j];
-  if (threadIdx.x < 32) {
+  // ---- merge the 2G partials: every thread loads its share at once ----
+  __shared__ MkPartial sh_part[kPickThreads / 32];
+  {
     SoftState st{-INFINITY, 0.0f};
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    for (int c = lane; c < 2 * p.G; c += 32) {
+    for (int c = threadIdx.x; c < 2 * p.G; c += kPickThreads) {
       const MkPartial o = p.part[(size_t)i * 2 * p.G + c];
       st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
       f |= o.flags;
@@ -483,12 +485,39 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
     }
     f = (int32_t)__reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
     if (lane == 0) {
-      sh_m = st.m;
-      sh_S = st.s;
-      sh_idx = kGreedy ? g.idx : best.idx;
-      sh_bad = (f || p.req_bad[i] || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
-                   ? 1 : 0;
+      MkPartial w{};
+      w.m = st.m;
+      w.s = st.s;
+      w.L = kGreedy ? g.v : best.L;
+      w.idx = kGreedy ? g.idx : best.idx;
+      w.M = best.M;
+      w.flags = f;
+      sh_part[threadIdx.x >> 5] = w;
     }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    SoftState st{-INFINITY, 0.0f};
+    MkKey best{INFINITY, 0.0f, INT_MAX};
+    ArgState g{-INFINITY, INT_MAX};
+    int32_t f = 0;
+    for (int w = 0; w < kPickThreads / 32; ++w) {
+      const MkPartial& o = sh_part[w];
+      st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
+      f |= o.flags;
+      if (kGreedy) {
+        const ArgState a{o.L, o.idx};
+        if (arg_better(a, g)) g = a;
+      } else {
+        const MkKey k{o.L, o.M, o.idx};
+        if (mk_better(k, best, p.c2)) best = k;
+      }
+    }
+    sh_m = st.m;
+    sh_S = st.s;
+    sh_idx = kGreedy ? g.idx : best.idx;
+    sh_bad = (f || p.req_bad[i] || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
+                 ? 1 : 0;
   }
   __syncthreads();
   const bool bad = sh_bad != 0;
