@@ -32,6 +32,15 @@ __device__ __forceinline__ unsigned long long position_key(float s, int k, int i
          ((unsigned long long)(0xFFFFu - (unsigned)k) << 16) | (unsigned long long)(0xFFFFu - (unsigned)i);
 }
 
+__device__ __forceinline__ unsigned long long lds_u64(uint32_t addr) {
+  unsigned long long v;
+  asm volatile("ld.shared.u64 %0, [%1];" : "=l"(v) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ void sts_u64(uint32_t addr, unsigned long long v) {
+  asm volatile("st.shared.u64 [%0], %1;" ::"r"(addr), "l"(v) : "memory");
+}
+
 // Inclusive block scan of one int64 value per thread (kAllocThreads threads).
 __device__ __forceinline__ long long block_inclusive_scan(long long x, long long* warp_tot) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -136,17 +145,20 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
   // ---- merge tree over the B sorted runs (descending) ----
   // Level l merges runs of L = L0 * 2^l keys; position e lies in run
   // (e / L0) >> l.  N <= 8192, so 32-bit indices suffice.
+  // The two key buffers by their shared-window addresses, so that every
+  // probe of the searches is a shared-memory load (ld.shared).
+  const uint32_t kbuf0 = (uint32_t)__cvta_generic_to_shared(sm.keys[0]);
+  const uint32_t kbuf1 = (uint32_t)__cvta_generic_to_shared(sm.keys[1]);
   int cur = 0;
   for (int lev = 0, L = L0; L < N; ++lev, L *= 2) {
-    const unsigned long long* in = sm.keys[cur];
-    unsigned long long* out = sm.keys[cur ^ 1];
+    const uint32_t in = cur ? kbuf1 : kbuf0, out = cur ? kbuf0 : kbuf1;
     for (int e = tid; e < N; e += kAllocThreads) {
       const int run = (e / L0) >> lev;
       const int start = run * L;
       const int pstart = (run ^ 1) * L;
-      const unsigned long long x = in[e];
+      const unsigned long long x = lds_u64(in + 8u * (uint32_t)e);
       if (pstart >= N) {  // unpaired last run: copied through
-        out[e] = x;
+        sts_u64(out + 8u * (uint32_t)e, x);
         continue;
       }
       const int plen = min(N, pstart + L) - pstart;
@@ -154,10 +166,10 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
       int lo = 0, hi = plen;
       while (lo < hi) {
         const int mid = (lo + hi) >> 1;
-        if (in[pstart + mid] > x) lo = mid + 1;
+        if (lds_u64(in + 8u * (uint32_t)(pstart + mid)) > x) lo = mid + 1;
         else hi = mid;
       }
-      out[min(start, pstart) + (e - start) + lo] = x;
+      sts_u64(out + 8u * (uint32_t)(min(start, pstart) + (e - start) + lo), x);
     }
     __syncthreads();
     cur ^= 1;
