@@ -410,7 +410,10 @@ int spec_draft(const void* logits, int logits_dtype, int B, int K, int V, float 
  * k = 0..K-1, with x_0 the last committed token,
  *   b_k = W1[x_k] W2,  q_k = softmax((U_k + b_k) / tau')  (tau' = tau, or 1),
  *   x_{k+1} ~ q_k by the two-level race at position pos_base + k + 1
- *   (purposes SPEC_PURPOSE_DRAFT / _IN_BLOCK), argmax at tau == 0;
+ *   over blocks of 64 consecutive entries (spec_draft races blocks of 256;
+ *   each is an exact draw from q_k; purposes SPEC_PURPOSE_DRAFT / _IN_BLOCK,
+ *   block b's level-1 variate is word b % 4 of sub-counter b / 4),
+ *   argmax at tau == 0;
  *   c_{k+1} = q_k(x_{k+1}); scores as spec_draft.
  * The bias of all B requests is one [B, r] x [r, V] contraction per position,
  * run on the tensor cores (tcgen05, fp32 accumulation): q, c and the row

@@ -77,6 +77,7 @@
 #define OR_PURPOSE_DRAFT 4u          /* the drafter's draw: block variates */
 #define OR_PURPOSE_DRAFT_IN_BLOCK 5u /* the drafter's draw: entry variates */
 #define OR_RACE_BLOCK 256
+#define OR_MARKOV_BLOCK 64 /* the Markov head's draw races blocks of 64 entries */
 
 /* ------------------------------------------------------------------------ */
 /* Element access.  bf16 is the upper half of an IEEE binary32 word.        */
@@ -177,13 +178,14 @@ double oracle_race_exponential(uint64_t seed, uint64_t request,
  * none).  Returns y, or -1 if every weight is zero. */
 static int two_level_race_with(const double* w, int V, uint64_t seed,
                                uint64_t request, uint64_t position,
-                               uint32_t pb, uint32_t pe, double* race_out) {
-  const int nb = (V + OR_RACE_BLOCK - 1) / OR_RACE_BLOCK;
+                               uint32_t pb, uint32_t pe, int block,
+                               double* race_out) {
+  const int nb = (V + block - 1) / block;
   double b1k = INFINITY, b2k = INFINITY;
   int b1 = -1, b2 = -1;
   for (int b = 0; b < nb; ++b) {
     double W = 0.0;
-    for (int v = b * OR_RACE_BLOCK; v < V && v < (b + 1) * OR_RACE_BLOCK; ++v)
+    for (int v = b * block; v < V && v < (b + 1) * block; ++v)
       W += w[v];
     if (!(W > 0.0)) continue;
     double key = race_exponential_with(seed, request, position, pb, (uint32_t)b) / W;
@@ -202,7 +204,7 @@ static int two_level_race_with(const double* w, int V, uint64_t seed,
   for (int pass = 0; pass < 2; ++pass) {
     int b = pass == 0 ? b1 : b2;
     if (b < 0) continue;
-    for (int v = b * OR_RACE_BLOCK; v < V && v < (b + 1) * OR_RACE_BLOCK; ++v) {
+    for (int v = b * block; v < V && v < (b + 1) * block; ++v) {
       if (!(w[v] > 0.0)) continue;
       double key = race_exponential_with(seed, request, position, pe, (uint32_t)v) / w[v];
       if (key < yk[pass]) {
@@ -237,7 +239,7 @@ static int two_level_race(const double* w, int V, uint64_t seed,
                           uint64_t request, uint64_t position,
                           double* race_out) {
   return two_level_race_with(w, V, seed, request, position, OR_PURPOSE_SAMPLE,
-                             OR_PURPOSE_SAMPLE_IN_BLOCK, race_out);
+                             OR_PURPOSE_SAMPLE_IN_BLOCK, OR_RACE_BLOCK, race_out);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -546,7 +548,7 @@ int oracle_draft_request(const void* logits, int dtype, int K, int V, double tau
     } else {
       for (int v = 0; v < V; ++v) w[v] = row_prob(row, dtype, v, tc, m, S);
       z = two_level_race_with(w, V, seed, request, (uint64_t)(pos_base + k + 1), OR_PURPOSE_DRAFT,
-                              OR_PURPOSE_DRAFT_IN_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
+                              OR_PURPOSE_DRAFT_IN_BLOCK, OR_RACE_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
     }
     if (z < 0) {
       bad = 1;
@@ -578,7 +580,9 @@ int oracle_draft_request(const void* logits, int dtype, int K, int V, double tau
 /* U_k of each position get the first-order bias b_k = W1[x_{k-1}] W2 of the */
 /* previously drawn token (x_0 the last committed token), and               */
 /* q_k = softmax((U_k + b_k) / tau').  Draws, confidences, scores and the    */
-/* bad-input rule as in oracle_draft_request, position by position.          */
+/* bad-input rule as in oracle_draft_request, position by position, except   */
+/* that the race's blocks hold 64 entries (the two-level race is an exact    */
+/* draw for any block size; this one matches the Markov kernel's tiles).     */
 /*   U [K, V] of dtype; W1 [V, r] and W2 [r, V] bf16 bits (uint16).          */
 /* ------------------------------------------------------------------------ */
 static double bf16_value(uint16_t h) {
@@ -631,7 +635,7 @@ int oracle_markov_request(const void* U, int dtype, const uint16_t* W1, const ui
     } else {
       for (int v = 0; v < V; ++v) w[v] = exp(l[v] / tc - m) / S;
       z = two_level_race_with(w, V, seed, request, (uint64_t)(pos_base + k + 1), OR_PURPOSE_DRAFT,
-                              OR_PURPOSE_DRAFT_IN_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
+                              OR_PURPOSE_DRAFT_IN_BLOCK, OR_MARKOV_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
     }
     if (z < 0) {
       bad = 1;

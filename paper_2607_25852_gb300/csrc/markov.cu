@@ -43,7 +43,8 @@ constexpr int kMkRows = 128;        // MMA M: request rows (rows >= B are zero)
 constexpr int kMkTile = 128;        // MMA N: vocabulary rows of W2^T per tile
 constexpr int kMkAtomK = 64;        // bf16 along K per 128-byte swizzle atom
 constexpr int kMkAtomBytes = 128 * 128;  // one atom of 128 rows x 128 bytes
-constexpr int kMkEpiWarps = 8;      // two per TMEM lane quarter, taking alternate race blocks
+constexpr int kMkEpiWarps = 8;      // two per TMEM lane quarter, taking alternate tiles
+constexpr int kMkBlock = 64;        // race block of this sampler (two per tile)
 constexpr int kMkThreads = 32 * (2 + kMkEpiWarps);  // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr int kMkMaxR = 256;
 constexpr int kMkSlots = 4;         // accumulators: (smem stage) x (epilogue half)
@@ -70,7 +71,7 @@ struct MarkovLaunch {
   const int64_t* pos_base;
   const int32_t* x0;
   __nv_bfloat16* E;  // [128, r]: W1 at the previous drafts
-  MkPartial* part;   // [B][2G]: one per epilogue half of each bias CTA
+  MkPartial* part;   // [B][G][4]: per bias CTA, per epilogue half and column half
   int G;
   uint32_t* req_bad;  // [B]
   int32_t* drafts;
@@ -233,15 +234,22 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   __shared__ int abort_flag;
   volatile int& abort_sh = abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nb = (p.V + kRaceBlock - 1) / kRaceBlock;
-  const int my_blocks = nb > (int)blockIdx.x ? (nb - 1 - (int)blockIdx.x) / p.G + 1 : 0;
-  const int T = 2 * my_blocks;                 // tiles: two halves per race block
-  // epilogue warps with at least one request row
-  const int n_epi = (p.B + 31) / 32;
+  const int ntiles = (p.V + kMkTile - 1) / kMkTile;
+  const int T = ntiles > (int)blockIdx.x ? (ntiles - 1 - (int)blockIdx.x) / p.G + 1 : 0;  // tile t: blockIdx.x + t G
+  // Epilogue warps: TMEM lane quarter q = warp % 4, half eh = the tiles with
+  // t % 2 == eh.  With B <= 64 the operand's rows 64..127 repeat rows 0..63,
+  // so every request row sits in two quarters: quarters 0-1 take a tile's
+  // columns 0..63 and quarters 2-3 its columns 64..127, and all four SM
+  // sub-partitions share the epilogue.  With B > 64 a warp takes its 32 rows
+  // over all 128 columns.
+  const bool dup = p.B <= 64;
   const bool epi = warp >= 2;
-  const int q = warp & 3;                      // TMEM lane quarter of this warp
-  const int eh = (warp - 2) >> 2;              // epilogue half: the race blocks j with j % 2 == eh
-  const bool epi_active = epi && 32 * q < p.B;
+  const int q = warp & 3;
+  const int eh = (warp - 2) >> 2;
+  const int row_q = dup ? (q & 1) : q;       // the quarter of request rows this warp serves
+  const int col_half = dup ? (q >> 1) : 0;   // with dup: columns [64 col_half, 64 col_half + 64)
+  const bool epi_active = epi && 32 * row_q < p.B;
+  const int n_epi = dup ? (p.B > 32 ? 4 : 2) : (p.B + 31) / 32;  // readers of each tile
 
   // E and the partials are read and written by the kernels around this one
   pdl_wait_prerequisites();
@@ -281,7 +289,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           break;
         }
         if (abort_sh) break;
-        const int v0 = ((int)blockIdx.x + (t >> 1) * p.G) * kRaceBlock + (t & 1) * kMkTile;
+        const int v0 = ((int)blockIdx.x + t * p.G) * kMkTile;
         mbar_expect_tx(&bar_full[s], (uint32_t)(nk * kMkAtomBytes));
         for (int a = 0; a < nk; ++a)
           tma_load_2d(sB + (s * nk + a) * kMkAtomBytes, &tmW, a * kMkAtomK, v0, &bar_full[s]);
@@ -321,105 +329,99 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     __syncwarp();
   } else if (epi_active) {
     // ---- epilogue: one request row per thread ----
-    const int row = 32 * q + lane;
+    const int row = 32 * row_q + lane;
     const bool valid = row < p.B;
     const size_t urow = ((size_t)(valid ? row : 0) * p.K + p.step) * (size_t)p.V;
     const long long pos = valid ? __ldg(reinterpret_cast<const long long*>(p.pos_base) + row) : 0;
     const uint32_t position = (uint32_t)(pos + p.step + 1);
     const uint64_t req = valid ? __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + row) : 0;
     const uint64_t seed = valid ? __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + row) : 0;
+    const int nblk = dup ? 1 : 2;            // race blocks of a tile this warp takes
+    const int blk0 = dup ? col_half : 0;
     SoftState st{-INFINITY, 0.0f};
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t flags = 0;
-    SoftState half{-INFINITY, 0.0f};  // the current race block's two halves
     bool aborted = false;
-    // a tile's 128 entries of U (bf16), loaded one tile ahead of their use
-    auto load_u = [&](int t, uint4 (&w)[16]) {
-      const int v0 = ((int)blockIdx.x + (t >> 1) * p.G) * kRaceBlock + (t & 1) * kMkTile;
+    uint4 uw[16];
+    for (int t = eh; t < T; t += 2) {
+      const int slot = t & 3;
+      const int v0 = ((int)blockIdx.x + t * p.G) * kMkTile;
+      // the warp's columns of U (bf16), fetched before the accumulator wait
 #pragma unroll
       for (int h = 0; h < 16; ++h) {
-        const int v = v0 + 8 * h;
+        if (h >= 8 * nblk) break;
+        const int v = v0 + kMkBlock * blk0 + 8 * h;
         if (valid && p.u_vec && v + 8 <= p.V) {
-          w[h] = ldg_stream(p.U + urow + v);
+          uw[h] = ldg_stream(p.U + urow + v);
         } else {
           uint32_t e[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j)
             e[j] = (valid && v + j < p.V) ? (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p.U) + urow + v + j)
                                           : 0xFF80u;  // -inf past V
-          w[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
+          uw[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
         }
       }
-    };
-    uint4 uw[16];
-    for (int t = 0; t < T; ++t) {
-      if (((t >> 1) & 1) != eh) continue;  // the other half's race block
-      const int slot = t & 3;
-      const int b = (int)blockIdx.x + (t >> 1) * p.G;
-      const int v0 = b * kRaceBlock + (t & 1) * kMkTile;
-      load_u(t, uw);  // issued before the accumulator wait
       const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(&bar_mma[slot], (uint32_t)((t >> 2) & 1), p.status));
       if (!ok) {
         aborted = true;
         break;
       }
       tc_fence_after();
-      // the tile's 4 chunks of 32 columns, each merged online: its max (and
-      // first argmax) and its sum relative to that max
-      SoftState tile{-INFINITY, 0.0f};
+      for (int cb = 0; cb < nblk; ++cb) {
+        const int bcol = kMkBlock * (blk0 + cb);  // the race block's first column in the tile
+        const int b = (v0 + bcol) / kMkBlock;
+        SoftState blk{-INFINITY, 0.0f};
 #pragma unroll
-      for (int ch = 0; ch < kMkTile / 32; ++ch) {
-        float l[32];
-        tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(slot * kMkTile + 32 * ch), l);
-        float cmax = -INFINITY;
+        for (int ch = 0; ch < kMkBlock / 32; ++ch) {
+          float l[32];
+          tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(slot * kMkTile + bcol + 32 * ch), l);
+          float cmax = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const uint4& w4 = uw[(32 * ch + k) >> 3];
-          const int e = k & 7;
-          const uint32_t word = e < 2 ? w4.x : e < 4 ? w4.y : e < 6 ? w4.z : w4.w;
-          l[k] += (e & 1) ? bf16_hi(word) : bf16_lo(word);  // -inf past V (U reads -inf there, the bias is 0)
-          cmax = fmaxf(cmax, l[k]);
+          for (int k = 0; k < 32; ++k) {
+            const uint4& w4 = uw[(kMkBlock * cb + 32 * ch + k) >> 3];
+            const int e = k & 7;
+            const uint32_t word = e < 2 ? w4.x : e < 4 ? w4.y : e < 6 ? w4.z : w4.w;
+            l[k] += (e & 1) ? bf16_hi(word) : bf16_lo(word);  // -inf past V (U reads -inf there, the bias is 0)
+            cmax = fmaxf(cmax, l[k]);
+          }
+          if (!valid) continue;
+          if (cmax == INFINITY) flags |= 1;
+          if (kGreedy && cmax > -INFINITY && (g.idx == INT_MAX || cmax > g.v || (cmax == g.v && v0 + bcol + 32 * ch < g.idx))) {
+            int first = INT_MAX;
+#pragma unroll
+            for (int k = 31; k >= 0; --k)
+              if (l[k] == cmax) first = v0 + bcol + 32 * ch + k;
+            if (g.idx == INT_MAX || cmax > g.v || first < g.idx) g = ArgState{cmax, first};
+          }
+          if (cmax > -INFINITY && cmax < INFINITY) {
+            const float M2 = cmax * p.c2;
+            float cs = 0.0f;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) cs += ex2_approx(__fmaf_rn(l[k], p.c2, -M2));
+            if (cs != cs) flags |= 1;  // a NaN entry
+            else blk = mk_merge(blk, SoftState{cmax, cs}, p.c2);
+          } else if (cmax != cmax) {
+            flags |= 1;
+          }
         }
         if (!valid) continue;
-        if (cmax == INFINITY) flags |= 1;
-        if (kGreedy && cmax > -INFINITY && (g.idx == INT_MAX || cmax > g.v)) {
-          int first = INT_MAX;
-#pragma unroll
-          for (int k = 31; k >= 0; --k)
-            if (l[k] == cmax) first = v0 + 32 * ch + k;
-          g = ArgState{cmax, first};
-        }
-        if (cmax > -INFINITY && cmax < INFINITY) {
-          const float M2 = cmax * p.c2;
-          float cs = 0.0f;
-#pragma unroll
-          for (int k = 0; k < 32; ++k) cs += ex2_approx(__fmaf_rn(l[k], p.c2, -M2));
-          if (cs != cs) flags |= 1;  // a NaN entry
-          else tile = mk_merge(tile, SoftState{cmax, cs}, p.c2);
-        } else if (cmax != cmax) {
-          flags |= 1;
+        // the race block is complete
+        st = mk_merge(st, blk, p.c2);
+        if (!kGreedy && blk.m > -INFINITY && blk.s > 0.0f && blk.s == blk.s) {
+          const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)(b >> 2)), (uint32_t)seed,
+                                  (uint32_t)(seed >> 32));
+          const uint32_t word = (b & 3) == 0 ? rq.x : (b & 3) == 1 ? rq.y : (b & 3) == 2 ? rq.z : rq.w;
+          const float E = -log1pf(-((float)race_m(word) * 0x1p-24f));
+          const MkKey cand{mk_lg2(E) - mk_lg2(blk.s), blk.m, b};
+          if (mk_better(cand, best, p.c2)) best = cand;
         }
       }
       // the accumulator is read: the MMA may overwrite it
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar_free[slot]);
-      if (!valid) continue;
-      half = mk_merge(half, tile, p.c2);
-      if ((t & 1) == 1 || t == T - 1) {
-        // the race block is complete
-        st = mk_merge(st, half, p.c2);
-        if (!kGreedy && half.m > -INFINITY && half.s > 0.0f && half.s == half.s) {
-          const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)(b >> 2)), (uint32_t)seed,
-                                  (uint32_t)(seed >> 32));
-          const uint32_t word = (b & 3) == 0 ? rq.x : (b & 3) == 1 ? rq.y : (b & 3) == 2 ? rq.z : rq.w;
-          const float E = -log1pf(-((float)race_m(word) * 0x1p-24f));
-          const MkKey cand{mk_lg2(E) - mk_lg2(half.s), half.m, b};
-          if (mk_better(cand, best, p.c2)) best = cand;
-        }
-        half = SoftState{-INFINITY, 0.0f};
-      }
     }
     if (valid && !aborted) {
       MkPartial o{};
@@ -429,7 +431,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       o.idx = kGreedy ? g.idx : best.idx;
       o.M = best.M;
       o.flags = flags;
-      p.part[(size_t)row * 2 * p.G + 2 * blockIdx.x + eh] = o;
+      MkPartial* dstp = p.part + ((size_t)row * p.G + blockIdx.x) * 4 + 2 * eh;
+      dstp[col_half] = o;
+      if (!dup) {  // this warp covered both column halves
+        MkPartial none{};
+        none.m = -INFINITY;
+        none.L = kGreedy ? -INFINITY : INFINITY;
+        none.idx = INT_MAX;
+        dstp[1] = none;
+      }
     }
   }
   tc_fence_before();
@@ -454,15 +464,15 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
   const int lane = threadIdx.x & 31;
   pdl_wait_prerequisites();
   for (int j = threadIdx.x; j < p.r; j += kPickThreads) sh_e[j] = p.E[(size_t)i * p.r + j];
-  // ---- merge the 2G partials: every thread loads its share at once ----
+  // ---- merge the 4G partials: every thread loads its share at once ----
   __shared__ MkPartial sh_part[kPickThreads / 32];
   {
     SoftState st{-INFINITY, 0.0f};
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    for (int c = threadIdx.x; c < 2 * p.G; c += kPickThreads) {
-      const MkPartial o = p.part[(size_t)i * 2 * p.G + c];
+    for (int c = threadIdx.x; c < 4 * p.G; c += kPickThreads) {
+      const MkPartial o = p.part[(size_t)i * 4 * p.G + c];
       st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
       f |= o.flags;
       if (kGreedy) {
@@ -535,7 +545,8 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
       // dot product in lane l.
       const int b = sh_idx;
       const int w_id = threadIdx.x >> 5;
-      const int v_base = b * kRaceBlock + 32 * w_id;
+      const int v_base = b * kMkBlock + 32 * w_id;
+      const bool in_block = 32 * w_id < kMkBlock;
       float part[32];
       {
         const bool has = 8 * lane < p.r;
@@ -545,8 +556,9 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
         uint4 w8[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j)
-          w8[j] = (has && v_base + j < p.V) ? __ldg(reinterpret_cast<const uint4*>(p.W2T + (size_t)(v_base + j) * p.r) + lane)
-                                            : make_uint4(0u, 0u, 0u, 0u);
+          w8[j] = (in_block && has && v_base + j < p.V)
+                      ? __ldg(reinterpret_cast<const uint4*>(p.W2T + (size_t)(v_base + j) * p.r) + lane)
+                      : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const uint32_t ww[4] = {w8[j].x, w8[j].y, w8[j].z, w8[j].w};
@@ -574,7 +586,7 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
       const int v = v_base + lane;
       KeyState e{INFINITY, INT_MAX};
       float l = -INFINITY;
-      if (v < p.V) {
+      if (in_block && v < p.V) {
         l = load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) + part[0];
         const float w = ex2_approx(__fmaf_rn(l, p.c2, -M2));
         const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
@@ -586,18 +598,21 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
         const uint32_t word = (v & 3) == 0 ? rw.x : (v & 3) == 1 ? rw.y : (v & 3) == 2 ? rw.z : rw.w;
         if (w > 0.0f) e = KeyState{race_key(race_m(word), w), v};
       }
-      sh_l[v - b * kRaceBlock] = l;
+      if (in_block) sh_l[v - b * kMkBlock] = l;
       e = cta_min_key(e, sh_red);
       if (threadIdx.x == 0) sh_idx = e.idx == INT_MAX ? -1 : e.idx;
       __syncthreads();
       z = sh_idx;
-      if (z >= 0) lz = sh_l[z - b * kRaceBlock];
+      if (z >= 0) lz = sh_l[z - b * kMkBlock];
     }
   }
   // the next position's operand row: W1 at this draft
   if (p.step + 1 < p.K)
-    for (int j = threadIdx.x; j < p.r; j += kPickThreads)
-      p.E[(size_t)i * p.r + j] = p.W1[(size_t)(bad || z < 0 ? 0 : z) * p.r + j];
+    for (int j = threadIdx.x; j < p.r; j += kPickThreads) {
+      const __nv_bfloat16 w = p.W1[(size_t)(bad || z < 0 ? 0 : z) * p.r + j];
+      p.E[(size_t)i * p.r + j] = w;
+      if (p.B <= 64) p.E[(size_t)(i + 64) * p.r + j] = w;  // the repeated rows
+    }
   if (threadIdx.x != 0) return;
   const size_t o = (size_t)i * p.K + p.step;
   if (bad || z < 0) {
@@ -639,7 +654,8 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
 // The first position's operand: W1 at the last committed tokens; rows past B
 // zero (the padding rows of the MMA).  One CTA per row of E.
 __global__ void __launch_bounds__(128) markov_begin_kernel(const MarkovLaunch p) {
-  const int i = blockIdx.x;
+  const int e = blockIdx.x;                 // row of E
+  const int i = p.B <= 64 ? (e & 63) : e;   // its request (rows 64..127 repeat 0..63 when B <= 64)
   pdl_wait_prerequisites();
   int x = 0;
   bool bad = true;
@@ -647,10 +663,10 @@ __global__ void __launch_bounds__(128) markov_begin_kernel(const MarkovLaunch p)
     x = __ldg(p.x0 + i);
     const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
     bad = x < 0 || x >= p.V || pos < 0 || pos + p.K > 0xFFFFFFFFLL;
-    if (threadIdx.x == 0) p.req_bad[i] = bad ? 1u : 0u;
+    if (threadIdx.x == 0 && e == i) p.req_bad[i] = bad ? 1u : 0u;
   }
   for (int j = threadIdx.x; j < p.r; j += blockDim.x)
-    p.E[(size_t)i * p.r + j] = (i < p.B && !bad) ? p.W1[(size_t)x * p.r + j] : __float2bfloat16(0.0f);
+    p.E[(size_t)e * p.r + j] = (i < p.B && !bad) ? p.W1[(size_t)x * p.r + j] : __float2bfloat16(0.0f);
 }
 
 // ---------------------------------------------------------------------------
@@ -689,11 +705,11 @@ struct MarkovGeometry {
 
 static MarkovGeometry markov_geometry(int B, int V, int r, int sms) {
   MarkovGeometry g{};
-  const int nb = (V + kRaceBlock - 1) / kRaceBlock;
-  g.G = std::max(1, std::min(sms, nb));
+  const int ntiles = (V + kMkTile - 1) / kMkTile;
+  g.G = std::max(1, std::min(sms, ntiles));
   g.e_off = 0;
   g.part_off = ((size_t)kMkRows * r * 2 + 255) / 256 * 256;
-  g.bad_off = g.part_off + ((size_t)sizeof(MkPartial) * B * 2 * g.G + 255) / 256 * 256;
+  g.bad_off = g.part_off + ((size_t)sizeof(MkPartial) * B * 4 * g.G + 255) / 256 * 256;
   g.bytes = g.bad_off + ((size_t)4 * B + 255) / 256 * 256;
   return g;
 }

@@ -115,18 +115,29 @@ def test_batch_sizes(B):
     assert compare_markov(g, o, U, W1, W2, x0, 1.0) <= max(1, B // 32)
 
 
-def test_zero_transition_matches_the_draft_step():
-    """W1 = 0: every bias vanishes and the draws are spec_draft's."""
+@pytest.mark.parametrize("tau", [0.0, 0.9])
+def test_zero_transition_matches_the_draft_step(tau):
+    """W1 = 0: every bias vanishes.  At tau = 0 the drafts and confidences are
+    spec_draft's; at tau > 0 the two races block the vocabulary differently
+    (64 against 256 entries, each an exact draw), so each confidence is
+    checked as q at the Markov draw."""
     import paper_2607_25852_gb300 as spec
     U, W1, W2, x0, seeds, rids, pos = _case(4, 5, 3000, 64, 8)
-    g = run_markov(U, torch.zeros_like(W1), W2, x0, 0.9, seeds, rids, pos)
-    ws = spec.draft_workspace(4, 5, 3000, DEV)
-    z = torch.zeros((4, 5), dtype=torch.int32, device=DEV)
-    c = torch.zeros((4, 5), device=DEV)
-    spec.spec_draft(U.to(DEV), 0.9, seeds.to(DEV), rids.to(DEV), pos.to(DEV), z, c, ws)
-    torch.cuda.synchronize()
-    assert np.array_equal(g["z"], z.cpu().numpy())
-    np.testing.assert_allclose(g["c"], c.cpu().numpy(), rtol=1e-5)
+    g = run_markov(U, torch.zeros_like(W1), W2, x0, tau, seeds, rids, pos)
+    assert g["status"] == 0
+    if tau == 0:
+        ws = spec.draft_workspace(4, 5, 3000, DEV)
+        z = torch.zeros((4, 5), dtype=torch.int32, device=DEV)
+        c = torch.zeros((4, 5), device=DEV)
+        spec.spec_draft(U.to(DEV), tau, seeds.to(DEV), rids.to(DEV), pos.to(DEV), z, c, ws)
+        torch.cuda.synchronize()
+        assert np.array_equal(g["z"], z.cpu().numpy())
+        np.testing.assert_allclose(g["c"], c.cpu().numpy(), rtol=1e-5)
+    else:
+        q = torch.softmax(U.double() / tau, dim=-1).numpy()
+        for i in range(4):
+            for k in range(5):
+                assert g["c"][i, k] == pytest.approx(q[i, k, g["z"][i, k]], rel=C_RTOL)
 
 
 def test_block_of_seven_drafts_full_vocabulary():
