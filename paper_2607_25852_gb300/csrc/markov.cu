@@ -47,7 +47,7 @@ constexpr int kMkEpiWarps = 8;      // two per TMEM lane quarter, taking alterna
 constexpr int kMkBlock = 64;        // race block of this sampler (two per tile)
 constexpr int kMkThreads = 32 * (2 + kMkEpiWarps);  // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr int kMkMaxR = 256;
-constexpr int kMkSlots = 4;         // accumulators: (smem stage) x (epilogue half)
+constexpr int kMkSlots = 4;         // accumulators: tile t in slot t % 4
 constexpr int kMkTmemCols = kMkSlots * kMkTile;  // 512 fp32 columns
 constexpr int kPickThreads = 256;
 
@@ -225,10 +225,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int nk = p.r / kMkAtomK;
   uint8_t* sA = smem;                          // nk atoms
   uint8_t* sB = smem + nk * kMkAtomBytes;      // 2 stages of nk atoms
-  // Tile t uses smem stage t & 1 and accumulator slot t & 3 (stage + 2 x the
-  // epilogue half of its race block), so that every waiter of a barrier sees
-  // its phases one after another (a parity wait two phases behind would
-  // alias).
+  // Tile t uses smem stage t & 1 and accumulator slot t & 3, so that every
+  // waiter of a barrier sees its phases one after another (a parity wait two
+  // phases behind would alias).
   __shared__ uint64_t bar_a, bar_full[2], bar_mma[kMkSlots], bar_free[kMkSlots];
   __shared__ uint32_t tmem_base_sh;
   __shared__ int abort_flag;
@@ -251,8 +250,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const bool epi_active = epi && 32 * row_q < p.B;
   const int n_epi = dup ? (p.B > 32 ? 4 : 2) : (p.B + 31) / 32;  // readers of each tile
 
-  // E and the partials are read and written by the kernels around this one
-  pdl_wait_prerequisites();
+  // The next kernel (this position's pick, 64 registers a thread) may take
+  // its place beside this CTA now and wait there for this grid to finish.
+  pdl_launch_dependents();
   if (threadIdx.x == 0) {
     mbar_init(&bar_a, 1);
     for (int s = 0; s < 2; ++s) mbar_init(&bar_full[s], 1);
@@ -279,12 +279,23 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     if (lane == 0 && T > 0) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmE)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
+      // W2^T and U are inputs of the whole draw, complete before its first
+      // kernel started: the first two tiles load while the previous
+      // position's pick runs.  E is that pick's output.
+      const int t_pre = T < 2 ? T : 2;
+      for (int t = 0; t < t_pre; ++t) {
+        const int v0 = ((int)blockIdx.x + t * p.G) * kMkTile;
+        mbar_expect_tx(&bar_full[t], (uint32_t)(nk * kMkAtomBytes));
+        for (int a = 0; a < nk; ++a)
+          tma_load_2d(sB + (t * nk + a) * kMkAtomBytes, &tmW, a * kMkAtomK, v0, &bar_full[t]);
+      }
+      pdl_wait_prerequisites();
       mbar_expect_tx(&bar_a, (uint32_t)(nk * kMkAtomBytes));
       for (int a = 0; a < nk; ++a) tma_load_2d(sA + a * kMkAtomBytes, &tmE, a * kMkAtomK, 0, &bar_a);
-      for (int t = 0; t < T; ++t) {
+      for (int t = t_pre; t < T; ++t) {
         const int s = t & 1;
         // the stage's previous tile (t - 2) has been consumed by its MMA
-        if (t >= 2 && !mbar_wait(&bar_mma[(t - 2) & 3], (uint32_t)(((t - 2) >> 2) & 1), p.status)) {
+        if (!mbar_wait(&bar_mma[(t - 2) & 3], (uint32_t)(((t - 2) >> 2) & 1), p.status)) {
           abort_sh = 1;
           break;
         }
@@ -363,6 +374,16 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           uw[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
         }
       }
+      // the warp's next tile of U, into L2 while this one is processed
+      if (valid && t + 2 < T) {
+        const int vn = ((int)blockIdx.x + (t + 2) * p.G) * kMkTile + kMkBlock * blk0;
+        const int ve = min(vn + kMkBlock * nblk, p.V) - 1;
+        if (vn < p.V)
+          for (int x = vn; x <= ve; x += 64) {
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(p.U + urow + x));
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(p.U + urow + min(x + 63, ve)));
+          }
+      }
       const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(&bar_mma[slot], (uint32_t)((t >> 2) & 1), p.status));
       if (!ok) {
         aborted = true;
@@ -423,6 +444,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar_free[slot]);
     }
+    pdl_wait_prerequisites();  // the previous position's pick has read the partials
     if (valid && !aborted) {
       MkPartial o{};
       o.m = st.m;
@@ -454,33 +476,60 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 // The draw of one position: merge, level 2, outputs, next E
 // ---------------------------------------------------------------------------
 template <bool kGreedy>
-__global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovLaunch p) {
+__global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const MarkovLaunch p) {
   __shared__ __align__(16) __nv_bfloat16 sh_e[kMkMaxR];
-  __shared__ float sh_l[kPickThreads];
+  __shared__ float sh_l[kMkBlock];
   __shared__ KeyState sh_red[kPickThreads / 32];
+  __shared__ MkPartial sh_part[kPickThreads / 32];
   __shared__ float sh_m, sh_S;
   __shared__ int sh_idx, sh_bad;
   const int i = blockIdx.x;
   const int lane = threadIdx.x & 31;
+  // inputs of the whole draw, read before the wait
+  const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
+  const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
+  const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+  // the next position's bias kernel may launch now: it prefetches its first
+  // W2^T tiles and waits for this grid before it reads E
+  pdl_launch_dependents();
   pdl_wait_prerequisites();
   for (int j = threadIdx.x; j < p.r; j += kPickThreads) sh_e[j] = p.E[(size_t)i * p.r + j];
-  // ---- merge the 4G partials: every thread loads its share at once ----
-  __shared__ MkPartial sh_part[kPickThreads / 32];
+  // ---- merge the 4G partials: each thread loads up to four before merging ----
   {
     SoftState st{-INFINITY, 0.0f};
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    for (int c = threadIdx.x; c < 4 * p.G; c += kPickThreads) {
-      const MkPartial o = p.part[(size_t)i * 4 * p.G + c];
-      st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
-      f |= o.flags;
-      if (kGreedy) {
-        const ArgState a{o.L, o.idx};
-        if (arg_better(a, g)) g = a;
-      } else {
-        const MkKey k{o.L, o.M, o.idx};
-        if (mk_better(k, best, p.c2)) best = k;
+    const int n = 4 * p.G;
+    const uint4* src = reinterpret_cast<const uint4*>(p.part + (size_t)i * n);
+    for (int c0 = threadIdx.x; c0 < n; c0 += 4 * kPickThreads) {
+      uint4 lo[4], hi[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + u * kPickThreads;
+        if (c < n) {
+          lo[u] = src[2 * c];
+          hi[u] = src[2 * c + 1];
+        } else {  // an empty partial
+          lo[u] = make_uint4(__float_as_uint(-INFINITY), 0u, __float_as_uint(kGreedy ? -INFINITY : INFINITY),
+                             (uint32_t)INT_MAX);
+          hi[u] = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float om = __uint_as_float(lo[u].x), os = __uint_as_float(lo[u].y);
+        const float oL = __uint_as_float(lo[u].z), oM = __uint_as_float(hi[u].x);
+        const int oidx = (int)lo[u].w;
+        st = soft_merge(st, SoftState{om, os}, p.c2);
+        f |= (int32_t)hi[u].y;
+        if (kGreedy) {
+          const ArgState a{oL, oidx};
+          if (arg_better(a, g)) g = a;
+        } else {
+          const MkKey k{oL, oM, oidx};
+          if (mk_better(k, best, p.c2)) best = k;
+        }
       }
     }
 #pragma unroll
@@ -506,28 +555,37 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {
+    // warp 0 merges the eight warps' results
     SoftState st{-INFINITY, 0.0f};
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    for (int w = 0; w < kPickThreads / 32; ++w) {
-      const MkPartial& o = sh_part[w];
-      st = soft_merge(st, SoftState{o.m, o.s}, p.c2);
-      f |= o.flags;
-      if (kGreedy) {
-        const ArgState a{o.L, o.idx};
-        if (arg_better(a, g)) g = a;
-      } else {
-        const MkKey k{o.L, o.M, o.idx};
-        if (mk_better(k, best, p.c2)) best = k;
-      }
+    if (lane < kPickThreads / 32) {
+      const MkPartial& o = sh_part[lane];
+      st = SoftState{o.m, o.s};
+      f = o.flags;
+      if (kGreedy) g = ArgState{o.L, o.idx};
+      else best = MkKey{o.L, o.M, o.idx};
     }
-    sh_m = st.m;
-    sh_S = st.s;
-    sh_idx = kGreedy ? g.idx : best.idx;
-    sh_bad = (f || p.req_bad[i] || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
-                 ? 1 : 0;
+#pragma unroll
+    for (int o = (kPickThreads / 32) / 2; o > 0; o >>= 1) {
+      st = soft_merge(st, SoftState{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)},
+                      p.c2);
+      const MkKey ok{__shfl_xor_sync(0xFFFFFFFFu, best.L, o), __shfl_xor_sync(0xFFFFFFFFu, best.M, o),
+                     __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
+      if (mk_better(ok, best, p.c2)) best = ok;
+      const ArgState og{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
+      if (arg_better(og, g)) g = og;
+    }
+    f = (int32_t)__reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
+    if (lane == 0) {
+      sh_m = st.m;
+      sh_S = st.s;
+      sh_idx = kGreedy ? g.idx : best.idx;
+      sh_bad = (f || p.req_bad[i] || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
+                   ? 1 : 0;
+    }
   }
   __syncthreads();
   const bool bad = sh_bad != 0;
@@ -538,29 +596,28 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
     if (kGreedy) {
       z = sh_idx;
     } else {
-      // level 2: the winning block's logits recomputed (U + E . W2^T row).
-      // Warp w takes entries 32w..32w+31 of the block; lane l multiplies the
+      // level 2: the winning block's 64 logits recomputed (U + E . W2^T row).
+      // Warp w takes entries 8w..8w+7 of the block; lane l multiplies the
       // r-slice 8l..8l+7 of each (one coalesced 16-byte load per entry, all
-      // issued at once), and a transposed butterfly leaves entry 32w + l's
-      // dot product in lane l.
+      // issued at once), and a transposed butterfly leaves entry 8w + l / 4's
+      // dot product in lanes 4 (l / 4)..4 (l / 4) + 3.
       const int b = sh_idx;
       const int w_id = threadIdx.x >> 5;
-      const int v_base = b * kMkBlock + 32 * w_id;
-      const bool in_block = 32 * w_id < kMkBlock;
-      float part[32];
+      const int v_base = b * kMkBlock + 8 * w_id;
+      float part[8];
       {
         const bool has = 8 * lane < p.r;
         uint4 e8 = make_uint4(0u, 0u, 0u, 0u);
         if (has) e8 = *reinterpret_cast<const uint4*>(sh_e + 8 * lane);
         const uint32_t ee[4] = {e8.x, e8.y, e8.z, e8.w};
-        uint4 w8[32];
+        uint4 w8[8];
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-          w8[j] = (in_block && has && v_base + j < p.V)
+        for (int j = 0; j < 8; ++j)
+          w8[j] = (has && v_base + j < p.V)
                       ? __ldg(reinterpret_cast<const uint4*>(p.W2T + (size_t)(v_base + j) * p.r) + lane)
                       : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
+        for (int j = 0; j < 8; ++j) {
           const uint32_t ww[4] = {w8[j].x, w8[j].y, w8[j].z, w8[j].w};
           float acc = 0.0f;
 #pragma unroll
@@ -571,9 +628,10 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
           part[j] = acc;
         }
       }
-      // transposed butterfly: 16 + 8 + 4 + 2 + 1 exchanges
+      // transposed butterfly over lane bits 4, 3, 2 (4 + 2 + 1 exchanges),
+      // then plain sums over bits 1 and 0
 #pragma unroll
-      for (int n = 32, o = 16; n > 1; n >>= 1, o >>= 1) {
+      for (int n = 8, o = 16; n > 1; n >>= 1, o >>= 1) {
         const bool hi = (lane & o) != 0;
 #pragma unroll
         for (int j = 0; j < n / 2; ++j) {
@@ -582,23 +640,22 @@ __global__ void __launch_bounds__(kPickThreads) markov_pick_kernel(const MarkovL
           part[j] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
         }
       }
-      // lane l now holds entry 32w + l (the halving kept the block of l's bits)
-      const int v = v_base + lane;
+      part[0] += __shfl_xor_sync(0xFFFFFFFFu, part[0], 2);
+      part[0] += __shfl_xor_sync(0xFFFFFFFFu, part[0], 1);
+      const int v = v_base + (lane >> 2);
+      const bool owner = (lane & 3) == 0;
       KeyState e{INFINITY, INT_MAX};
       float l = -INFINITY;
-      if (in_block && v < p.V) {
+      if (owner && v < p.V) {
         l = load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) + part[0];
         const float w = ex2_approx(__fmaf_rn(l, p.c2, -M2));
-        const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
-        const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
-        const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
         const uint4 rw = philox(draw_counter((uint32_t)(pos + p.step + 1), req, SPEC_PURPOSE_DRAFT_IN_BLOCK,
                                              (uint32_t)(v >> 2)),
                                 (uint32_t)seed, (uint32_t)(seed >> 32));
         const uint32_t word = (v & 3) == 0 ? rw.x : (v & 3) == 1 ? rw.y : (v & 3) == 2 ? rw.z : rw.w;
         if (w > 0.0f) e = KeyState{race_key(race_m(word), w), v};
       }
-      if (in_block) sh_l[v - b * kMkBlock] = l;
+      if (owner) sh_l[8 * w_id + (lane >> 2)] = l;
       e = cta_min_key(e, sh_red);
       if (threadIdx.x == 0) sh_idx = e.idx == INT_MAX ? -1 : e.idx;
       __syncthreads();
