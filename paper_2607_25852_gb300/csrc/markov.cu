@@ -358,13 +358,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     for (int t = eh; t < T; t += 2) {
       const int slot = t & 3;
       const int v0 = ((int)blockIdx.x + t * p.G) * kMkTile;
-      // the warp's columns of U (bf16), fetched before the accumulator wait
+      // the warp's columns of U (bf16), fetched before the accumulator wait.
+      // A lane reads 128 consecutive bytes of its own row in 16-byte loads;
+      // the loads allocate in L1, so each 32-byte sector crosses from L2 once.
 #pragma unroll
       for (int h = 0; h < 16; ++h) {
         if (h >= 8 * nblk) break;
         const int v = v0 + kMkBlock * blk0 + 8 * h;
         if (valid && p.u_vec && v + 8 <= p.V) {
-          uw[h] = ldg_stream(p.U + urow + v);
+          uw[h] = __ldg(reinterpret_cast<const uint4*>(p.U + urow + v));
         } else {
           uint32_t e[8];
 #pragma unroll
@@ -604,6 +606,16 @@ __global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const Mark
       const int b = sh_idx;
       const int w_id = threadIdx.x >> 5;
       const int v_base = b * kMkBlock + 8 * w_id;
+      const int v = v_base + (lane >> 2);
+      const bool owner = (lane & 3) == 0;
+      // the rows of W1 at the block's entries, into L2: one of them becomes
+      // the next position's E row (thread t: row t / 4, 128-byte line t % 4)
+      if (p.step + 1 < p.K) {
+        const int wv = b * kMkBlock + (threadIdx.x >> 2), line = threadIdx.x & 3;
+        if (wv < p.V && line < p.r / 64)
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(p.W1 + (size_t)wv * p.r + 64 * line));
+      }
+      const float u_v = (owner && v < p.V) ? load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) : 0.0f;
       float part[8];
       {
         const bool has = 8 * lane < p.r;
@@ -642,12 +654,10 @@ __global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const Mark
       }
       part[0] += __shfl_xor_sync(0xFFFFFFFFu, part[0], 2);
       part[0] += __shfl_xor_sync(0xFFFFFFFFu, part[0], 1);
-      const int v = v_base + (lane >> 2);
-      const bool owner = (lane & 3) == 0;
       KeyState e{INFINITY, INT_MAX};
       float l = -INFINITY;
       if (owner && v < p.V) {
-        l = load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) + part[0];
+        l = u_v + part[0];
         const float w = ex2_approx(__fmaf_rn(l, p.c2, -M2));
         const uint4 rw = philox(draw_counter((uint32_t)(pos + p.step + 1), req, SPEC_PURPOSE_DRAFT_IN_BLOCK,
                                              (uint32_t)(v >> 2)),
