@@ -147,3 +147,33 @@ def test_draft_workspace_and_argument_errors(lib):
     assert d(4, 4, 100, 1.0, stats=ctypes.c_void_p(20)) == 1     # row stats not 8-byte aligned
     assert d(4, 4, 100, 1.0, ws_bytes=8) == 2
     assert d(4, 4, 100, 1.0, ws=ctypes.c_void_p(264)) == 2
+
+
+def test_markov_workspace_and_argument_errors(lib):
+    """spec_markov_draft's shape, dtype, temperature, pointer and workspace
+    checks fail before any CUDA launch."""
+    import paper_2607_25852_gb300 as spec
+    ws_size = lib.spec_markov_workspace
+    for B, K, V, r in [(0, 7, 1000, 64), (129, 7, 1000, 64), (4, 0, 1000, 64), (4, 7, 0, 64), (4, 7, 1000, 32),
+                       (4, 7, 1000, 100), (4, 7, 1000, 320)]:
+        assert ws_size(B, K, V, r) == 0, (B, K, V, r)
+    n = ws_size(64, 7, 201088, 256)
+    assert n > 0 and n % 256 == 0 and n < (64 << 20)
+    assert ws_size(128, 7, 201088, 256) > n                        # partials scale with B
+    dummy = ctypes.c_void_p(16)                                    # never dereferenced: every call fails a check
+    stream = ctypes.c_void_p(0)
+
+    def d(B=4, K=3, V=1000, r=64, tau=1.0, dt=0, w1=dummy, w2=dummy, stats=None, ws=ctypes.c_void_p(256),
+          ws_bytes=1 << 24, U=dummy):
+        return lib.spec_markov_draft(U, dt, w1, w2, r, dummy, B, K, V, tau, dummy, dummy, dummy, dummy, dummy, None,
+                                     stats, None, ws, ws_bytes, stream)
+    assert d(B=0) == 1 and d(B=129) == 1 and d(K=0) == 1 and d(V=0) == 1
+    assert d(r=0) == 1 and d(r=96) == 1 and d(r=512) == 1
+    assert d(tau=-0.5) == 1 and d(tau=float("nan")) == 1 and d(tau=float("inf")) == 1
+    assert d(dt=1) == 1                                             # U must be bf16
+    assert d(U=None) == 1 and d(w1=None) == 1 and d(w2=None) == 1
+    assert d(w1=ctypes.c_void_p(24)) == 1 and d(w2=ctypes.c_void_p(40)) == 1   # 16-byte alignment
+    assert d(stats=ctypes.c_void_p(20)) == 1                        # row stats not 8-byte aligned
+    assert d(ws_bytes=8) == 2                                       # workspace too small
+    assert d(ws=ctypes.c_void_p(264)) == 2                          # workspace not 256-aligned
+    assert d(ws=None) == 2
