@@ -177,3 +177,33 @@ def test_markov_workspace_and_argument_errors(lib):
     assert d(ws_bytes=8) == 2                                       # workspace too small
     assert d(ws=ctypes.c_void_p(264)) == 2                          # workspace not 256-aligned
     assert d(ws=None) == 2
+
+
+def test_round_graph_and_pack_rows_argument_errors(lib):
+    """The graph helpers, spec_select_round and spec_pack_rows reject bad
+    arguments before any CUDA call."""
+    from paper_2607_25852_gb300 import _native
+    hdr = open(HEADER).read()
+    max_cand = int(re.search(r"#define SPEC_MAX_CANDIDATES\s+(\d+)", hdr).group(1))
+    max_drafts = int(re.search(r"#define SPEC_MAX_DRAFTS\s+(\d+)", hdr).group(1))
+    dummy = ctypes.c_void_p(16)                 # never dereferenced: every call fails a check
+    stream = ctypes.c_void_p(0)
+    assert lib.spec_graph_begin_capture(None) == 1          # the legacy stream cannot be captured
+    assert lib.spec_graph_end_capture(stream, 0, None) == 1
+    assert lib.spec_graph_launch(None, stream) == 1
+    assert lib.spec_graph_destroy(None) == 0                # destroying nothing is fine
+    cand = (ctypes.c_int32 * 2)(8, 16)
+    graphs_ok = (ctypes.c_void_p * 2)(16, 32)
+    graphs_hole = (ctypes.c_void_p * 2)(16, None)
+    sel = lambda chosen, M, c, g: lib.spec_select_round(chosen, M, c, g, None, None, stream)
+    assert sel(None, 2, cand, graphs_ok) == 1
+    assert sel(dummy, 0, cand, graphs_ok) == 1
+    assert sel(dummy, max_cand + 1, cand, graphs_ok) == 1
+    assert sel(dummy, 2, None, graphs_ok) == 1
+    assert sel(dummy, 2, cand, None) == 1
+    assert sel(dummy, 2, cand, graphs_hole) == 1            # every candidate needs a graph
+    pk = lambda src=dummy, rb=64, B=4, K=3, offs=dummy, dst=dummy, R=8: lib.spec_pack_rows(
+        src, rb, B, K, offs, dst, R, None, stream)
+    assert pk(src=None) == 1 and pk(dst=None) == 1 and pk(offs=None) == 1
+    assert pk(rb=0) == 1 and pk(B=0) == 1 and pk(K=-1) == 1 and pk(K=max_drafts + 1) == 1 and pk(R=0) == 1
+    assert _native.SIGNATURES["spec_pack_rows"][1][1] is ctypes.c_size_t
