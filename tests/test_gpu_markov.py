@@ -140,15 +140,16 @@ def test_zero_transition_matches_the_draft_step(tau):
                 assert g["c"][i, k] == pytest.approx(q[i, k, g["z"][i, k]], rel=C_RTOL)
 
 
-def test_block_of_seven_drafts_full_vocabulary():
-    """B = 64 requests, a block of 8 (K = 7 drafts), V = 201088, r = 256 at
-    tau = 1: eight requests through the oracle."""
+@pytest.mark.parametrize("tau", [1.0, 0.0])
+def test_block_of_seven_drafts_full_vocabulary(tau):
+    """B = 64 requests, a block of 8 (K = 7 drafts), V = 201088, r = 256
+    (the measured configuration): eight requests through the oracle."""
     U, W1, W2, x0, seeds, rids, pos = _case(64, 7, 201088, 256, 9, std=3.0, wstd=0.2)
-    g = run_markov(U, W1, W2, x0, 1.0, seeds, rids, pos)
+    g = run_markov(U, W1, W2, x0, tau, seeds, rids, pos)
     assert g["status"] == 0
     picks = [0, 9, 18, 27, 36, 45, 54, 63]
-    o = run_oracle_markov(U, W1, W2, x0, 1.0, seeds, rids, pos, requests=picks)
-    ties = compare_markov(g, o, U, W1, W2, x0, 1.0, requests=picks)
+    o = run_oracle_markov(U, W1, W2, x0, tau, seeds, rids, pos, requests=picks)
+    ties = compare_markov(g, o, U, W1, W2, x0, tau, requests=picks)
     print("markov full-size ties:", ties)
     assert ties <= 1
 
@@ -165,3 +166,15 @@ def test_bad_inputs_are_flagged_per_request():
     assert o["status"].tolist() == [oracle.ERR_BAD_INPUT] * 3 + [0]
     compare_markov(g, o, U, W1, W2, x0, 1.0)
     assert (g["s"][:3, 1:] == 0).all() and (g["s"][:3, 0] == 1).all()
+
+
+@pytest.mark.parametrize("B,r", [(65, 64), (100, 192), (7, 192)])
+def test_batches_past_the_repeated_rows_and_three_atom_rank(B, r):
+    """B = 65 and 100: the operand is not repeated, every lane quarter takes
+    its own rows over all columns (the last quarter part-filled); r = 192:
+    three K-atoms per tile."""
+    U, W1, W2, x0, seeds, rids, pos = _case(B, 3, 3000, r, 40 + B + r)
+    g = run_markov(U, W1, W2, x0, 0.9, seeds, rids, pos)
+    o = run_oracle_markov(U, W1, W2, x0, 0.9, seeds, rids, pos)
+    assert g["status"] == 0 and (o["status"] == 0).all()
+    assert compare_markov(g, o, U, W1, W2, x0, 0.9) <= max(1, B // 32)
