@@ -456,6 +456,11 @@ def run_ours(args):
             graph = {"error": f"{type(exc).__name__}: {exc}"[:300]}
 
     # ---- end to end through the same API with pinned host buffers ----
+    # The large inputs (logits, q, hidden rows) are read in place by the
+    # kernels when the device reaches the pinned buffers at the same address
+    # (NVLink-C2C on Grace-Blackwell); the small ones are copied.  The
+    # copy-engine variant (every input copied to device memory first) is
+    # measured too.
     e2e = None
     if not args.no_e2e:
         host = {k: getattr(wl, k).cpu().pin_memory() for k in
@@ -466,26 +471,43 @@ def run_ours(args):
         outs_host = [torch.empty_like(t, device="cpu").pin_memory() for t in (step.acc, step.tok, step.ctok, step.coff)]
         h2d = sum(v.numel() * v.element_size() for v in host.values())
         d2h = sum(t.numel() * t.element_size() for t in outs_host)
+        big = [k for k in ("logits", "q", "hidden") if k in host]
+        in_place_ok = all(step.spec.spec_pointer_device_readable(host[k]) for k in big)
 
-        def e2e_step():
+        def e2e_step(in_place):
+            x = dict(dev_in)
             for k, v in host.items():
-                dev_in[k].copy_(v, non_blocking=True)
-            step.run(dev_in)
+                if in_place and k in big:
+                    x[k] = v
+                else:
+                    dev_in[k].copy_(v, non_blocking=True)
+            step.run(x)
             for o, d in zip(outs_host, (step.acc, step.tok, step.ctok, step.coff)):
                 o.copy_(d, non_blocking=True)
 
-        for _ in range(2):
-            e2e_step()
-        torch.cuda.synchronize()
-        n_e2e = max(3, min(args.steps, 10))
-        barrier(dist)
-        t0 = time.perf_counter()
-        for _ in range(n_e2e):
-            e2e_step()
-        torch.cuda.synchronize()
-        el = max_over_ranks(dist, time.perf_counter() - t0, device)
-        e2e = {"value": world * R * n_e2e / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "steps": n_e2e, "ms_per_step": 1e3 * el / n_e2e}
+        def measure(in_place):
+            for _ in range(2):
+                e2e_step(in_place)
+            torch.cuda.synchronize()
+            n = max(3, min(args.steps, 10))
+            barrier(dist)
+            t0 = time.perf_counter()
+            for _ in range(n):
+                e2e_step(in_place)
+            torch.cuda.synchronize()
+            el = max_over_ranks(dist, time.perf_counter() - t0, device)
+            return world * R * n / el, 1e3 * el / n, n
+
+        v_copy, ms_copy, n_copy = measure(False)
+        if in_place_ok:
+            v, ms, n = measure(True)
+            how = "pinned host logits, q and hidden rows read in place by the kernels; small inputs copied"
+        else:
+            v, ms, n = v_copy, ms_copy, n_copy
+            how = "every input copied to device memory first"
+        e2e = {"value": v, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
+               "ms_per_step": ms, "h2d": how,
+               "copy_engine": {"value": v_copy, "ms_per_step": ms_copy}}
 
     if rank != 0:
         if dist is not None:

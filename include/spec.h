@@ -102,6 +102,18 @@ const char* spec_error_string(int code);
 int spec_version(void);
 
 /* ------------------------------------------------------------------------
+ * spec_pointer_device_readable -- 1 if the library's kernels may read `ptr`
+ * in place: device or managed memory, or host memory that the device reaches
+ * at the same address (pinned by cudaHostAlloc / cudaHostRegister under
+ * unified addressing).  0 otherwise (including when no device is present).
+ * Inputs marked "device or host-mapped" below may be such host memory: the
+ * kernels then read it over the CPU-GPU link (NVLink-C2C on Grace-Blackwell)
+ * with no staging copy.  No counterpart in the paper: a property of the
+ * hardware the library runs on.
+ * ---------------------------------------------------------------------- */
+int spec_pointer_device_readable(const void* ptr);
+
+/* ------------------------------------------------------------------------
  * spec_budget_from_ratios -- Eq. (dcut-budget), Section 4.2:
  *   T_m = max(B, ceil(num[m] / den[m] * B * (K + 1)))
  * in exact integer arithmetic, for M ratios (the paper's set is
@@ -176,16 +188,17 @@ int spec_allocate(const float* conf, int B, int K, const int32_t* cand_T,
  *           P(b*) = W_b / W and P(y | b*) = w_y / W_b.
  *   out_tokens[i] = z_1..z_a, y, then -1 up to K+1 entries.
  * Arguments
- *   logits          device [R, V] of logits_dtype, rows of request i at
- *                   row_offsets[i] .. row_offsets[i] + n_i.
+ *   logits          device or host-mapped [R, V] of logits_dtype, rows of
+ *                   request i at row_offsets[i] .. row_offsets[i] + n_i.
  *   row_offsets     device int32 [B+1] (from spec_allocate) or NULL, meaning
  *                   row_offsets[i] = i(K+1) and R = B(K+1).
  *   depth           device int32 [B] (n_i in [0, K]) or NULL meaning n_i = K.
  *                   If row_offsets is given, row_offsets[i+1] - row_offsets[i]
  *                   must equal n_i + 1 (else SPEC_ERR_BAD_INPUT for i).
  *   draft_tokens    device int32 [B, K] (z_{j+1} at [i][j]); may be NULL if K=0.
- *   q               device [B, K, V] of q_dtype (row j of request i is the
- *                   drafter's distribution of z_{j+1}, used as stored), or
+ *   q               device or host-mapped [B, K, V] of q_dtype (row j of
+ *                   request i is the drafter's distribution of z_{j+1}, used
+ *                   as stored), or
  *                   NULL: one-hot at the draft token.  Ignored when t == 0.
  *   temperature     t >= 0 and finite.
  *   seeds, request_ids  device uint64 [B]; pos_base device int64 [B]
@@ -257,7 +270,8 @@ int spec_verify_static(const void* logits, int logits_dtype, const int32_t* row_
  * Arguments
  *   accepted_len, out_tokens  device int32 [B], [B, K+1] (from spec_verify).
  *   row_offsets     device int32 [B+1] or NULL (= i(K+1)).
- *   hidden          device [R, H] of hidden_dtype, or NULL (tokens only).
+ *   hidden          device or host-mapped [R, H] of hidden_dtype, or NULL
+ *                   (tokens only).
  *   packed_tokens_out device int32 [B(K+1)] (entries past the total are
  *                   not written); commit_offsets_out device int32 [B+1];
  *   hidden_out      device [B(K+1), H] (worst case) or NULL.

@@ -42,6 +42,7 @@ __all__ = [
     "spec_shard_finish", "shard_workspace", "spec_draft_workspace", "spec_draft", "draft_workspace",
     "spec_graph_begin_capture", "spec_graph_end_capture", "spec_graph_launch", "spec_graph_destroy",
     "spec_select_round", "spec_pack_rows", "spec_markov_workspace", "spec_markov_draft", "markov_workspace",
+    "spec_pointer_device_readable",
 ]
 
 
@@ -93,6 +94,13 @@ def spec_version() -> int:
 
 def spec_error_string(code: int) -> str:
     return library().spec_error_string(code).decode()
+
+
+def spec_pointer_device_readable(t) -> bool:
+    """True if the library's kernels may read tensor t in place: device
+    memory, or pinned host memory mapped at the same address (read over the
+    CPU-GPU link with no staging copy)."""
+    return bool(library().spec_pointer_device_readable(_ptr(t)))
 
 
 def spec_budget_from_ratios(B: int, K: int, num, den):

@@ -17,6 +17,7 @@ _SZ = ctypes.c_size_t
 SIGNATURES = {
     "spec_error_string": (ctypes.c_char_p, [_I]),
     "spec_version": (_I, []),
+    "spec_pointer_device_readable": (_I, [_P]),
     "spec_budget_from_ratios": (_I, [_I, _I, _P, _P, _I, _P]),
     "spec_allocate_workspace": (_SZ, [_I, _I, _I]),
     "spec_allocate": (_I, [_P, _I, _I, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),

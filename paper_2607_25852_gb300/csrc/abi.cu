@@ -52,6 +52,17 @@ const char* spec_error_string(int code) {
 
 int spec_version(void) { return SPEC_ABI_VERSION; }
 
+int spec_pointer_device_readable(const void* ptr) {
+  if (!ptr) return 0;
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    cudaGetLastError();  // clear the error this query may leave
+    return 0;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return 1;
+  return a.type == cudaMemoryTypeHost && a.devicePointer == ptr ? 1 : 0;
+}
+
 int spec_budget_from_ratios(int B, int K, const int32_t* num, const int32_t* den, int M,
                             int32_t* cand_T_out) {
   if (B < 1 || K < 0 || M < 1 || !num || !den || !cand_T_out) return SPEC_ERR_INVALID_ARG;

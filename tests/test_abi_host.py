@@ -207,3 +207,11 @@ def test_round_graph_and_pack_rows_argument_errors(lib):
     assert pk(src=None) == 1 and pk(dst=None) == 1 and pk(offs=None) == 1
     assert pk(rb=0) == 1 and pk(B=0) == 1 and pk(K=-1) == 1 and pk(K=max_drafts + 1) == 1 and pk(R=0) == 1
     assert _native.SIGNATURES["spec_pack_rows"][1][1] is ctypes.c_size_t
+
+
+def test_pointer_readability_without_a_device(lib):
+    """No pointer is promised device-readable when the query fails (no GPU
+    here) or the pointer is NULL."""
+    assert lib.spec_pointer_device_readable(None) == 0
+    buf = ctypes.create_string_buffer(64)
+    assert lib.spec_pointer_device_readable(ctypes.cast(buf, ctypes.c_void_p)) in (0, 1)
