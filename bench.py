@@ -501,13 +501,21 @@ def run_ours(args):
         v_copy, ms_copy, n_copy = measure(False)
         if in_place_ok:
             v, ms, n = measure(True)
-            how = "pinned host logits, q and hidden rows read in place by the kernels; small inputs copied"
+            # what crosses the link in place: every logits row, the q row at
+            # each rejection and the q(z) sectors, the committed hidden rows,
+            # and the small inputs that are copied
+            ab = algorithmic_bytes(wl, step.acc.cpu().numpy())
+            small_bytes = sum(t.numel() * t.element_size() for k, t in host.items() if k not in big)
+            h2d_moved = (ab["logits"] + ab["q_rows"] + (wl.B * wl.K * 32 if wl.q is not None else 0)
+                         + ab["commit"] // 2 + small_bytes)
+            how = ("pinned host logits, q and hidden rows read in place by the kernels (only the bytes the "
+                   "method reads cross the link); small inputs copied")
         else:
-            v, ms, n = v_copy, ms_copy, n_copy
+            v, ms, n, h2d_moved = v_copy, ms_copy, n_copy, h2d
             how = "every input copied to device memory first"
-        e2e = {"value": v, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n,
-               "ms_per_step": ms, "h2d": how,
-               "copy_engine": {"value": v_copy, "ms_per_step": ms_copy}}
+        e2e = {"value": v, "unit": UNIT, "h2d_bytes_per_step": h2d_moved, "d2h_bytes_per_step": d2h, "steps": n,
+               "ms_per_step": ms, "h2d": how, "host_input_bytes_per_step": h2d,
+               "copy_engine": {"value": v_copy, "ms_per_step": ms_copy, "h2d_bytes_per_step": h2d}}
 
     if rank != 0:
         if dist is not None:
