@@ -9,23 +9,29 @@
 // 5th-generation tensor cores.
 //
 //   markov_bias_kernel  persistent, one CTA per SM.  Warp 0 loads by TMA the
-//                       operand E_k (128 x r, requests padded with zero rows)
-//                       once and then tiles of W2^T (128 vocabulary rows x r,
+//                       operand E_k (128 x r; with B <= 64 rows 64..127
+//                       repeat rows 0..63, other rows past B are zero) once,
+//                       and the CTA's tiles of W2^T (128 vocabulary rows x r,
 //                       128-byte swizzle), double-buffered.  Warp 1 issues
 //                       tcgen05.mma (M = 128, N = 128, K = 16, bf16 -> fp32)
-//                       into four TMEM accumulators.  Eight epilogue warps (two
-//                       per TMEM lane quarter, alternate race blocks) read the
-//                       accumulator rows (tcgen05.ld, one request per thread),
-//                       add U_k, and per race block of 256 entries
-//                       form the block's max and sum, its level-1 race key
-//                       (or its argmax at tau = 0) and the row's softmax
-//                       statistics.  Each epilogue half of a CTA writes one
-//                       partial per request.
+//                       into four TMEM accumulators.  Eight epilogue warps
+//                       (two per TMEM lane quarter, alternate tiles) read the
+//                       accumulator rows (tcgen05.ld, one request per
+//                       thread; with the repeated rows, one column half of
+//                       each tile per quarter pair), add U_k, and per race
+//                       block of 64 entries form the block's max and sum, its
+//                       level-1 race key (or its argmax at tau = 0) and the
+//                       row's softmax statistics: four partials per request
+//                       and CTA.
 //   markov_pick_kernel  one CTA per request: merges the partials, recomputes
-//                       the winning block's 256 logits and draws inside it
+//                       the winning block's 64 logits and draws inside it
 //                       (level 2), writes the draft, its confidence and the
 //                       row statistics, and gathers W1 at the draft into E for
 //                       the next position.
+//
+// Consecutive kernels overlap through programmatic dependent launch: each
+// triggers its dependent at entry, and the bias kernel loads its first W2^T
+// tiles before it waits for the previous position's pick.
 //
 // Every mbarrier wait is bounded (about a second): a wait that gives up sets
 // SPEC_ERR_TIMEOUT, the kernel stops issuing work, waits (bounded) for what
