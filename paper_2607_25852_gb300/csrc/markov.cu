@@ -256,8 +256,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const bool epi_active = epi && 32 * row_q < p.B;
   const int n_epi = dup ? (p.B > 32 ? 4 : 2) : (p.B + 31) / 32;  // readers of each tile
 
-  // The next kernel (this position's pick, 64 registers a thread) may take
-  // its place beside this CTA now and wait there for this grid to finish.
+  // The next kernel (this position's pick) may launch now; its CTAs do not
+  // fit beside a bias CTA (registers), so they start as bias CTAs exit.
   pdl_launch_dependents();
   if (threadIdx.x == 0) {
     mbar_init(&bar_a, 1);
