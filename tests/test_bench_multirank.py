@@ -79,3 +79,27 @@ def test_reference_arm_under_torchrun_prints_once():
     line = json.loads(lines[0])
     assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle"
+
+
+class _Wl:
+    """The fields of a workload that the byte accounting reads."""
+    def __init__(self, B, K, V, H, dtype="bf16", q=True, hidden=True):
+        self.B, self.K, self.V, self.H, self.dtype = B, K, V, H, dtype
+        self.q = object() if q else None
+        self.hidden = object() if hidden else None
+
+
+def test_algorithmic_bytes_count_what_the_method_reads():
+    """Every logits row once, a q row per rejecting request, the q(z)/l(z)
+    sectors, the committed hidden rows read and written, the small arrays."""
+    import numpy as np
+    B, K, V, H = 4, 3, 1000, 64
+    acc = np.array([3, 0, 1, 3])                    # two requests reject (a < K)
+    ab = bench.algorithmic_bytes(_Wl(B, K, V, H), acc)
+    assert ab["logits"] == B * (K + 1) * V * 2
+    assert ab["q_rows"] == 2 * V * 2
+    assert ab["gathers"] == B * K * 2 * 32
+    assert ab["commit"] == 2 * int((acc + 1).sum()) * H * 2
+    assert ab["total"] == ab["logits"] + ab["q_rows"] + ab["gathers"] + ab["commit"] + ab["small"]
+    none = bench.algorithmic_bytes(_Wl(B, K, V, H, dtype="f32", q=False, hidden=False), acc)
+    assert none["logits"] == B * (K + 1) * V * 4 and none["q_rows"] == 0 and none["commit"] == 0
