@@ -4,11 +4,15 @@
 // At most SPEC_MAX_ALLOC_POSITIONS = 8192 positions, so the whole problem fits
 // in shared memory.  Every position (i, k) becomes one 64-bit key
 //   bits(s_{i,k}) << 32 | (0xFFFF - k) << 16 | (0xFFFF - i)
-// whose descending order is the allocator's total order: s >= 0, so the fp32
-// bit pattern is monotone in s; then shallower k first (the paper's tie rule);
+// whose descending order is the allocator's total order: s >= +0 (a -0
+// confidence is taken as +0), so the fp32 bit pattern is monotone in s; then
+// shallower k first (the paper's tie rule);
 // then lower request index.  Keys are unique.
 //
-// Because s_{i,k} is non-increasing in k, each request's K+1 keys already form
+// Batches of at most 1024 requests and 1024 draft positions take
+// allocate_small_kernel (below): a bitonic sort of the draft keys alone.
+// Larger batches take allocate_kernel:
+// because s_{i,k} is non-increasing in k, each request's K+1 keys already form
 // a run sorted in descending order.  A merge tree of ceil(log2 B) levels sorts
 // the B runs: at every level each key finds its place in the merged pair by
 // one binary search in the partner run.  An inclusive scan of floor(s * 2^40)
@@ -136,6 +140,9 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
         sh_bad = 1;
         c = 0.0f;
       }
+      // -0 passes the range check and equals 0, but its sign bit would put
+      // its key above every positive score: -0 + 0 = +0 drops the sign.
+      c = __fadd_rn(c, 0.0f);
       s = __fmul_rn(s, c);
       sm.keys[0][i * L0 + k] = position_key(s, k, i);
     }
@@ -264,7 +271,184 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
   if (tid == 0 && sh_bad) report(p.status, SPEC_ERR_BAD_INPUT);
 }
 
+// ---------------------------------------------------------------------------
+// Batches of at most 1024 requests and 1024 draft positions (B * K)
+// ---------------------------------------------------------------------------
+// Every bonus position (k = 0) has the largest score (s = 1) and the smallest
+// k, so it ranks above every draft position, and the bonus positions rank
+// among themselves by request index.  The global order is therefore the B
+// bonus positions, then the B * K draft keys sorted; only the latter need a
+// sort.  One draft key per thread, sorted by a bitonic network over 1024 slots
+// (padding key 0 ranks below every real key, whose k field is nonzero):
+// partners within a warp exchange by shuffles, others through shared memory,
+// one barrier per such stage.  The keep depths then follow from the sorted
+// ranks without atomics: draft (i, k) in the top T - B, with (i, k + 1) not,
+// ends request i's kept prefix.
+constexpr int kSmallSlots = kAllocThreads;
+
+__device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long x, int o) {
+  const unsigned lo = __shfl_xor_sync(0xFFFFFFFFu, (unsigned)x, o);
+  const unsigned hi = __shfl_xor_sync(0xFFFFFFFFu, (unsigned)(x >> 32), o);
+  return ((unsigned long long)hi << 32) | lo;
+}
+
+__global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const AllocLaunch p) {
+  __shared__ float sh_conf[2 * kSmallSlots];               // [i][k] at i * (K | 1) + k
+  __shared__ int32_t sh_drafts[kSmallSlots];
+  __shared__ int32_t sh_last[kSmallSlots];
+  __shared__ long long sh_pos[kSmallSlots];
+  __shared__ unsigned long long sh_x[2][kSmallSlots];      // sort exchanges, then prefix sums / depths
+  __shared__ int32_t sh_rank[kSmallSlots];                 // sorted rank of draft (i, k) at i * K + k - 1
+  __shared__ long long warp_tot[32];
+  __shared__ int sh_best_c, sh_bad;
+  const int B = p.B, K = p.K, NK = B * K, CS = K | 1;
+  const int tid = threadIdx.x;
+  if (tid == 0) sh_bad = 0;
+  // The next kernel (the streaming pass) may launch now: it waits for this
+  // one's completion before it reads the depths and row offsets.
+  pdl_launch_dependents();
+
+  // ---- every global input in one round trip ----
+  if (tid < NK) {
+    const int i = tid / K;
+    sh_conf[tid + i * (CS - K)] = p.conf[tid];
+    sh_drafts[tid] = p.drafts[tid];
+  }
+  if (tid < B) {
+    sh_last[tid] = p.last_tokens[tid];
+    sh_pos[tid] = p.pos_base[tid];
+  }
+  __syncthreads();
+
+  // ---- Eq. (dcut-score): fp32 prefix products, request i in thread i ----
+  if (tid < B) {
+    const float* ci = sh_conf + tid * CS;
+    float s = 1.0f;
+    for (int k = 1; k <= K; ++k) {
+      float c = ci[k - 1];
+      if (!(c >= 0.0f && c <= 1.0f)) {
+        sh_bad = 1;
+        c = 0.0f;
+      }
+      c = __fadd_rn(c, 0.0f);  // -0 counts as +0 (its sign bit would break the key order)
+      s = __fmul_rn(s, c);
+      sh_x[0][tid * K + (k - 1)] = position_key(s, k, tid);
+    }
+  }
+  __syncthreads();
+
+  // ---- bitonic sort of the draft keys, descending ----
+  unsigned long long x = tid < NK ? sh_x[0][tid] : 0ull;
+  int buf = 1;
+#pragma unroll 1
+  for (int k = 2; k <= kSmallSlots; k <<= 1) {
+#pragma unroll 1
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      unsigned long long y;
+      if (j >= 32) {
+        sh_x[buf][tid] = x;
+        __syncthreads();
+        y = sh_x[buf][tid ^ j];
+        buf ^= 1;
+      } else {
+        y = shfl_xor_u64(x, j);
+      }
+      // blocks of k alternate direction (descending first); the lower index
+      // of a pair keeps the larger key in a descending block
+      const bool take_max = ((tid & k) == 0) == ((tid & j) == 0);
+      x = take_max ? (x > y ? x : y) : (x < y ? x : y);
+    }
+  }
+  // x: the draft key of rank tid (tid < NK)
+  const int xi = 0xFFFF - (int)(x & 0xFFFFull);
+  const int xk = 0xFFFF - (int)((x >> 16) & 0xFFFFull);
+  if (tid < NK) sh_rank[xi * K + (xk - 1)] = tid;
+
+  // ---- inclusive scan of floor(s * 2^40) over the sorted draft keys ----
+  const long long q40 = tid < NK ? (long long)__float2ll_rd(__uint_as_float((unsigned)(x >> 32)) * 0x1p40f) : 0;
+  const long long incl = block_inclusive_scan(q40, warp_tot);  // its barriers also end the sort's reads
+  long long* prefix = reinterpret_cast<long long*>(sh_x[0]);
+  prefix[tid] = incl;
+  __syncthreads();
+
+  // ---- Eq. (dcut-select): first maximiser of U / cost ----
+  if (tid < 32) {
+    double best_obj = -INFINITY;
+    int best_c = INT_MAX;
+    for (int c = tid; c < p.M; c += 32) {
+      const int td = p.cand_T[c] - B;  // draft positions kept at this budget
+      const long long Uq = ((long long)B << 40) + (td > 0 ? prefix[td - 1] : 0);
+      const double U = (double)Uq * 0x1p-40;
+      if (p.utility_out) p.utility_out[c] = U;
+      const double obj = U / p.cand_cost[c];
+      if (obj > best_obj) {  // c increases along the lane's loop
+        best_obj = obj;
+        best_c = c;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const double ob = __shfl_xor_sync(0xFFFFFFFFu, best_obj, o);
+      const int cb = __shfl_xor_sync(0xFFFFFFFFu, best_c, o);
+      if (ob > best_obj || (ob == best_obj && cb < best_c)) {
+        best_obj = ob;
+        best_c = cb;
+      }
+    }
+    if (tid == 0) sh_best_c = best_c == INT_MAX ? 0 : best_c;
+  }
+  int* depth = reinterpret_cast<int*>(sh_x[1]);
+  int* offsets = depth + kSmallSlots;
+  if (tid < B) depth[tid] = 0;
+  __syncthreads();
+  const int T = p.cand_T[sh_best_c];
+  const int TD = T - B;
+
+  // ---- keep depths: the last kept draft of each request ----
+  if (tid < NK && tid < TD) {
+    const bool next_kept = xk < K && sh_rank[xi * K + xk] < TD;
+    if (!next_kept) depth[xi] = xk;
+  }
+  __syncthreads();
+
+  // ---- row offsets: exclusive scan of (n_i + 1) ----
+  const int cnt = tid < B ? depth[tid] + 1 : 0;
+  const long long rincl = block_inclusive_scan((long long)cnt, warp_tot);
+  if (tid < B) {
+    offsets[tid] = (int)(rincl - cnt);
+    p.row_offsets_out[tid] = (int)(rincl - cnt);
+    p.depth_out[tid] = cnt - 1;
+  }
+  if (tid == 0) {
+    p.row_offsets_out[B] = T;  // sum of (n_i + 1): the T kept positions
+    *p.chosen_T_out = T;
+  }
+  __syncthreads();
+
+  // ---- dense packing of the kept prefixes ----
+  if (tid < B) {
+    p.packed_tokens_out[offsets[tid]] = sh_last[tid];
+    p.packed_pos_out[offsets[tid]] = sh_pos[tid];
+  }
+  if (tid < NK && tid < TD) {
+    const int row = offsets[xi] + xk;
+    p.packed_tokens_out[row] = sh_drafts[xi * K + (xk - 1)];
+    p.packed_pos_out[row] = sh_pos[xi] + xk;
+  }
+  for (int r = T + tid; r < B * (K + 1); r += kAllocThreads) {
+    p.packed_tokens_out[r] = -1;
+    p.packed_pos_out[r] = -1;
+  }
+  if (tid == 0 && sh_bad) report(p.status, SPEC_ERR_BAD_INPUT);
+}
+
+bool allocate_is_small(int B, int K) { return B <= kSmallSlots && (long long)B * K <= kSmallSlots; }
+
 cudaError_t launch_allocate(const AllocLaunch& p, cudaStream_t stream) {
+  if (allocate_is_small(p.B, p.K)) {
+    allocate_small_kernel<<<1, kAllocThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+  }
   const size_t smem = allocate_smem_bytes(p.B, p.K);
   cudaError_t err = cudaFuncSetAttribute(allocate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);

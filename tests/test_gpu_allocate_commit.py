@@ -85,6 +85,29 @@ def test_random_allocations(B, K):
         assert_alloc_equal(g, r)
 
 
+@pytest.mark.parametrize("B,K", [(4, 3), (64, 16), (300, 7)])
+def test_negative_zero_confidences(B, K):
+    """-0 confidences (the value 0, sign bit set) rank as zero scores: the
+    allocation is bit-exact with the oracle at T = B, T = B(K+1) and random
+    budgets, and no depth is ever negative."""
+    rng = np.random.default_rng(B + K)
+    conf = rng.uniform(size=(B, K)).astype(np.float32)
+    mask = rng.random((B, K)) < 0.3
+    conf[mask] = np.float32(-0.0)
+    conf[0, :] = np.float32(-0.0)
+    assert np.signbit(conf[0, 0])
+    N = B * (K + 1)
+    Ts = sorted(set(int(x) for x in rng.integers(B, N + 1, size=6)) | {B, N})
+    costs = list(rng.uniform(0.5, 3.0, len(Ts)))
+    for cand in [[B], [N], Ts]:
+        cc = costs[:len(cand)] if cand is Ts else [1.0]
+        g = gpu_allocate(torch.as_tensor(conf), cand, cc)
+        r = oracle.allocate(conf, cand, cc)
+        assert int(g["status"][0]) == 0 and r["status"] == 0
+        assert_alloc_equal(g, r)
+        assert (g["depth"] >= 0).all()
+
+
 def test_sixty_four_candidates():
     """The most candidates a call takes (SPEC_MAX_CANDIDATES), with tied scores."""
     rng = np.random.default_rng(64)

@@ -89,6 +89,30 @@ def test_ties_go_to_shallower_positions_then_lower_requests():
     assert d[4].tolist() == [K] * B
 
 
+def test_negative_zero_confidence_counts_as_zero():
+    """-0 is the value 0 (Eq. dcut-score then gives s = 0): an allocation with
+    -0 confidences equals the one with +0 everywhere, and the zero scores
+    rank after every positive score with the tie rule (shallower k, then
+    lower request)."""
+    B, K = 4, 3
+    pos = np.array([[0.9, -0.0, 0.5], [-0.0, 0.7, 0.7], [0.6, 0.6, 0.6], [-0.0, -0.0, -0.0]], np.float32)
+    assert np.signbit(pos[1, 0]) and pos[1, 0] == 0.0
+    plus = np.abs(pos)
+    N = B * (K + 1)
+    Ts = np.array([B, B + 3, B + 5, B + 7, N], np.int32)
+    a = oracle.allocate(pos, Ts, np.ones(len(Ts)))
+    b = oracle.allocate(plus, Ts, np.ones(len(Ts)))
+    assert a["status"] == 0 and b["status"] == 0
+    for k in ("depth", "row_offsets", "packed_tokens", "packed_pos", "utility", "all_depths"):
+        assert np.array_equal(a[k], b[k]), k
+    d = a["all_depths"]
+    assert d[0].tolist() == [0, 0, 0, 0]                     # the bonus positions first
+    assert d[1].tolist() == [1, 0, 2, 0]                     # s = 0.9, 0.6, 0.36
+    assert d[2].tolist() == [1, 1, 3, 0]                     # 0.216, then the first zero: request 1, k = 1
+    assert d[3].tolist() == [2, 1, 3, 1]                     # zeros: request 3 at k = 1, then request 0 at k = 2
+    assert d[4].tolist() == [K] * B
+
+
 def test_expected_advance_and_monotone_utility():
     rng = np.random.default_rng(5)
     B, K = 8, 6
