@@ -132,6 +132,22 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
                 const uint64_t* request_ids, const int64_t* pos_base, int32_t* accepted_len_out,
                 int32_t* out_tokens, float* p_draft_out, float* row_stats_out, int32_t* status,
                 void* ws, size_t ws_bytes, cudaStream_t stream) {
+  return spec::verify_impl(logits, logits_dtype, row_offsets, depth, draft_tokens, q, q_dtype, B, K, V,
+                           temperature, seeds, request_ids, pos_base, accepted_len_out, out_tokens,
+                           p_draft_out, row_stats_out, status, ws, ws_bytes, stream, nullptr, nullptr);
+}
+
+}  // extern "C"
+
+// spec_verify with a hook that runs once every host-side check has passed,
+// immediately before the first launch (nullptr: none).  A hook that fails
+// makes the call return SPEC_ERR_CUDA with nothing launched.
+int spec::verify_impl(const void* logits, int logits_dtype, const int32_t* row_offsets, const int32_t* depth,
+                      const int32_t* draft_tokens, const void* q, int q_dtype, int B, int K, int V,
+                      float temperature, const uint64_t* seeds, const uint64_t* request_ids,
+                      const int64_t* pos_base, int32_t* accepted_len_out, int32_t* out_tokens,
+                      float* p_draft_out, float* row_stats_out, int32_t* status, void* ws, size_t ws_bytes,
+                      cudaStream_t stream, cudaError_t (*pre_launch)(void*, cudaStream_t), void* hook_ctx) {
   NvtxRange range("spec_verify");
   cudaEvent_t ev_before = g_profile_before, ev_after = g_profile_after;
   g_profile_before = g_profile_after = nullptr;
@@ -188,8 +204,11 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
     const bool q_ok = p.q == nullptr || (reinterpret_cast<uintptr_t>(p.q) % 16 == 0 && (V * qsize) % 16 == 0);
     p.vec_s = V % 8 == 0 && reinterpret_cast<uintptr_t>(logits) % 16 == 0 && (V * esize) % 16 == 0 && q_ok;
   }
+  if (pre_launch && pre_launch(hook_ctx, stream) != cudaSuccess) return SPEC_ERR_CUDA;
   return spec::launch_verify(p, stream, ev_before, ev_after) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
+
+extern "C" {
 
 int spec_commit(const int32_t* accepted_len, const int32_t* out_tokens, const int32_t* row_offsets,
                 const void* hidden, int hidden_dtype, int B, int K, int H,

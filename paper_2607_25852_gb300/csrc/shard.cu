@@ -130,8 +130,15 @@ static inline size_t round256(size_t x) { return (x + 255) / 256 * 256; }
 static ShardGeometry shard_geometry(int B, int K, int Vs) {
   const VerifyGeometry g = verify_geometry(B, K, Vs);
   ShardGeometry s;
-  s.NC = g.NC;
-  s.chunk = g.chunk;
+  // Streaming pass: aim for ~4096 (row, chunk) CTAs, each a whole number of
+  // load rounds (256 threads x 8 16-byte vectors = 16384 bf16 entries), so
+  // that only the last chunk of a row ends in a partial round.
+  const long long R = (long long)B * (K + 1);
+  long long nc = (4096 + R - 1) / R;
+  nc = std::max(1LL, std::min(nc, std::max(1LL, (long long)Vs / 16384)));
+  const long long chunk = ((Vs + nc - 1) / nc + 16383) / 16384 * 16384;
+  s.NC = (int)((Vs + chunk - 1) / chunk);  // every chunk non-empty
+  s.chunk = (int)chunk;
   s.quads_s = g.chunk_s / kRaceQuad;
   // a shard of Vs columns spans at most ceil(Vs / 1024) + 1 quads
   const long long nq_max = (Vs + kRaceQuad - 1) / kRaceQuad + 1;

@@ -240,4 +240,13 @@ cudaError_t launch_verify(const VerifyLaunch& p, cudaStream_t stream, cudaEvent_
 cudaError_t launch_allocate(const AllocLaunch& p, cudaStream_t stream);
 cudaError_t launch_commit(const CommitLaunch& p, cudaStream_t stream);
 
+// spec_verify's host checks and launches, with an optional hook that runs
+// after every check has passed and before anything is launched.
+int verify_impl(const void* logits, int logits_dtype, const int32_t* row_offsets, const int32_t* depth,
+                const int32_t* draft_tokens, const void* q, int q_dtype, int B, int K, int V, float temperature,
+                const uint64_t* seeds, const uint64_t* request_ids, const int64_t* pos_base,
+                int32_t* accepted_len_out, int32_t* out_tokens, float* p_draft_out, float* row_stats_out,
+                int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream,
+                cudaError_t (*pre_launch)(void*, cudaStream_t), void* hook_ctx);
+
 }  // namespace spec

@@ -89,3 +89,35 @@ def test_static_scratch_rejects_shapes_beyond_its_size():
         spec.spec_verify_static(logits, o["tok"], None, B, K, V, 1.0, dummy, dummy, dummy,
                                 o["acc"], o["tok"])
     assert e.value.code == spec.ERR_TOO_LARGE
+
+
+def test_static_scratch_over_a_sequence_of_shapes():
+    """Shapes that change from call to call: the counters and records move
+    inside the shared array, and a smaller call's counters start where a
+    larger call left its partials.  Every call must still match spec_verify
+    with a fresh caller workspace."""
+    seq = [(65536, 64, 16, 1.0, True), (4097, 5, 3, 0.8, False), (65536, 64, 16, 1.0, True),
+           (20000, 8, 5, 0.0, False), (4097, 5, 3, 0.8, False), (333, 3, 0, 1.3, False)]
+    for n, (V, B, K, t, dense_q) in enumerate(seq):
+        x = _inputs(V, B, K, t, dense_q, seed=V + B + n)
+        want = _run(x, static=False)
+        got = _run(x, static=True)
+        assert int(got["status"][0]) == 0 and int(want["status"][0]) == 0, (V, B, K)
+        assert np.array_equal(got["acc"], want["acc"]), (V, B, K)
+        assert np.array_equal(got["tok"], want["tok"]), (V, B, K)
+        np.testing.assert_allclose(got["pdr"], want["pdr"], rtol=P_RTOL, atol=1e-30)
+        np.testing.assert_allclose(got["rst"], want["rst"], rtol=P_RTOL, atol=P_RTOL)
+
+
+def test_static_scratch_argument_error_leaves_the_next_call_intact():
+    """A call rejected on the host (negative temperature) queues nothing; the
+    call after it is still correct."""
+    x = _inputs(4097, 5, 3, 0.8, False, seed=77)
+    o = _outputs(5, 3)
+    with pytest.raises(spec.SpecError) as e:
+        spec.spec_verify_static(x["logits"], x["drafts"], None, 5, 3, 4097, -1.0, x["seeds"], x["request_ids"],
+                                x["pos_base"], o["acc"], o["tok"])
+    assert e.value.code == spec.ERR_INVALID_ARG
+    want = _run(x, static=False)
+    got = _run(x, static=True)
+    assert np.array_equal(got["acc"], want["acc"]) and np.array_equal(got["tok"], want["tok"])
