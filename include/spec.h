@@ -49,6 +49,7 @@
  *   (lo32(position), lo32(request_id_i), hi32(request_id_i), purpose<<28 | sub)
  *   SPEC_PURPOSE_ACCEPT: sub = 0; u = (word0 >> 8) * 2^-24 in [0, 1)
  *   SPEC_PURPOSE_SAMPLE:          sub = b >> 2; block variate E_b from word[b & 3]
+ *                                 (block b = entries [256 b, 256 b + 256))
  *   SPEC_PURPOSE_SAMPLE_IN_BLOCK: sub = v >> 2; entry variate E'_v from word[v & 3]
  *   SPEC_PURPOSE_DRAFT, SPEC_PURPOSE_DRAFT_IN_BLOCK: the same two variates
  *                  for spec_draft's draw of the drafts
@@ -82,6 +83,10 @@ typedef enum {
 } spec_err;
 
 typedef enum { SPEC_BF16 = 0, SPEC_F32 = 1 } spec_dtype;
+
+/* Entries per level-1 block of the two-level exponential race, the same for
+ * every draw of the library (verification, spec_draft, spec_markov_draft). */
+#define SPEC_RACE_BLOCK 256
 
 #define SPEC_PURPOSE_ACCEPT 1u
 #define SPEC_PURPOSE_SAMPLE 2u
@@ -240,12 +245,16 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
  *   - Returns SPEC_ERR_TOO_LARGE, launching nothing, when
  *     spec_verify_workspace(B, K, V) exceeds SPEC_STATIC_SCRATCH_BYTES
  *     (4 MiB holds about 260,000 16-byte row-chunk partials; B=64, K=16,
- *     V=201088 needs 86 KB).
+ *     V=201088 needs spec_verify_workspace(64, 16, 201088) bytes, about
+ *     80 KB).
  *   - The first call on a device looks up the array's device address (once
- *     per device, with that device current); make that first call before
- *     any stream capture.
+ *     per device and CUDA context, with that device current); make that
+ *     first call before any stream capture.  A new context on the device
+ *     (after cudaDeviceReset, say) is looked up again on its first call.
  *   - Every call on a device shares the one array, which keeps the previous
- *     call's contents; each call clears the part that must start at zero.
+ *     call's contents; each call clears the part that must start at zero,
+ *     on `stream`, after every argument check has passed (a call that
+ *     returns an error has queued nothing).
  *     Calls that overlap on the GPU (concurrent streams, or several host
  *     threads) race on the array and give wrong results: serialise them.
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
@@ -423,11 +432,10 @@ int spec_draft(const void* logits, int logits_dtype, int B, int K, int V, float 
  * Eq. dspark-markov; the block factorisation Eq. ar-factorization): for
  * k = 0..K-1, with x_0 the last committed token,
  *   b_k = W1[x_k] W2,  q_k = softmax((U_k + b_k) / tau')  (tau' = tau, or 1),
- *   x_{k+1} ~ q_k by the two-level race at position pos_base + k + 1
- *   over blocks of 64 consecutive entries (spec_draft races blocks of 256;
- *   each is an exact draw from q_k; purposes SPEC_PURPOSE_DRAFT / _IN_BLOCK,
- *   block b's level-1 variate is word b % 4 of sub-counter b / 4),
- *   argmax at tau == 0;
+ *   x_{k+1} ~ q_k by spec_draft's two-level race (blocks of
+ *   SPEC_RACE_BLOCK entries, purposes SPEC_PURPOSE_DRAFT / _IN_BLOCK) at
+ *   position pos_base + k + 1, argmax at tau == 0: with W1 = 0 the draws
+ *   are spec_draft's on the same U;
  *   c_{k+1} = q_k(x_{k+1}); scores as spec_draft.
  * The bias of all B requests is one [B, r] x [r, V] contraction per position,
  * run on the tensor cores (tcgen05, fp32 accumulation): q, c and the row

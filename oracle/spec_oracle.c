@@ -20,7 +20,7 @@
  *     correctness" paragraph: dense packing of the unequal prefixes, and the
  *     deterministic-draft, target-only protocol (one-hot q).
  *
- * Readings where the paper is silent (each is listed in the design notes):
+ * Readings where the paper is silent:
  *   - verification rule: standard speculative sampling (accept draft z with
  *     probability min(1, p(z)/q(z)); on the first rejection draw from
  *     norm(max(0, p - q)); if every draft is accepted draw the bonus from p);
@@ -33,7 +33,11 @@
  *     b* = argmin_{W_b > 0} E_b / W_b is drawn first, then the entry
  *     y = argmin_{v in b*, w_v > 0} E'_v / w_v (ties to the lowest index at
  *     both levels).  Each level is an exact draw (P(b*) = W_b / W,
- *     P(y | b*) = w_y / W_b), so P(y) = w_y / W;
+ *     P(y | b*) = w_y / W_b), so P(y) = w_y / W.  Every draw (verification,
+ *     the drafter's step and the Markov head's step) uses these 256-entry
+ *     blocks: an exact draw is all the method asks for, and a draw costs
+ *     V / 256 + 256 variates, near the minimum 2 sqrt(V) of V / b + b for the
+ *     vocabularies of 128K-201K entries the method serves;
  *   - temperature 0 is the longest argmax-matching prefix plus the argmax of
  *     the first unmatched row (ties to lowest index);
  *   - allocator scores are fp32 products taken in order k = 1..K (the
@@ -76,8 +80,7 @@
 #define OR_PURPOSE_SAMPLE_IN_BLOCK 3u
 #define OR_PURPOSE_DRAFT 4u          /* the drafter's draw: block variates */
 #define OR_PURPOSE_DRAFT_IN_BLOCK 5u /* the drafter's draw: entry variates */
-#define OR_RACE_BLOCK 256
-#define OR_MARKOV_BLOCK 64 /* the Markov head's draw races blocks of 64 entries */
+#define OR_RACE_BLOCK 256 /* entries per level-1 block, the same for every draw */
 
 /* ------------------------------------------------------------------------ */
 /* Element access.  bf16 is the upper half of an IEEE binary32 word.        */
@@ -580,9 +583,9 @@ int oracle_draft_request(const void* logits, int dtype, int K, int V, double tau
 /* U_k of each position get the first-order bias b_k = W1[x_{k-1}] W2 of the */
 /* previously drawn token (x_0 the last committed token), and               */
 /* q_k = softmax((U_k + b_k) / tau').  Draws, confidences, scores and the    */
-/* bad-input rule as in oracle_draft_request, position by position, except   */
-/* that the race's blocks hold 64 entries (the two-level race is an exact    */
-/* draw for any block size; this one matches the Markov kernel's tiles).     */
+/* bad-input rule as in oracle_draft_request, position by position: the     */
+/* same two-level race (blocks of OR_RACE_BLOCK entries, purposes DRAFT and  */
+/* DRAFT_IN_BLOCK), so that with W1 = 0 the draw is the draft step's.        */
 /*   U [K, V] of dtype; W1 [V, r] and W2 [r, V] bf16 bits (uint16).          */
 /* ------------------------------------------------------------------------ */
 static double bf16_value(uint16_t h) {
@@ -635,7 +638,7 @@ int oracle_markov_request(const void* U, int dtype, const uint16_t* W1, const ui
     } else {
       for (int v = 0; v < V; ++v) w[v] = exp(l[v] / tc - m) / S;
       z = two_level_race_with(w, V, seed, request, (uint64_t)(pos_base + k + 1), OR_PURPOSE_DRAFT,
-                              OR_PURPOSE_DRAFT_IN_BLOCK, OR_MARKOV_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
+                              OR_PURPOSE_DRAFT_IN_BLOCK, OR_RACE_BLOCK, race_out ? race_out + (size_t)k * 9 : NULL);
     }
     if (z < 0) {
       bad = 1;

@@ -18,15 +18,16 @@
 //                       (two per TMEM lane quarter, alternate tiles) read the
 //                       accumulator rows (tcgen05.ld, one request per
 //                       thread; with the repeated rows, one column half of
-//                       each tile per quarter pair), add U_k, and per race
-//                       block of 64 entries form the block's max and sum, its
-//                       level-1 race key (or its argmax at tau = 0) and the
-//                       row's softmax statistics: four partials per request
-//                       and CTA.
-//   markov_pick_kernel  one CTA per request: merges the partials, recomputes
-//                       the winning block's 64 logits and draws inside it
-//                       (level 2), writes the draft, its confidence and the
-//                       row statistics, and gathers W1 at the draft into E for
+//                       each tile per quarter pair), add U_k, and per
+//                       64-column sub-block write its max and sum; they also
+//                       keep the row's softmax statistics (or its argmax at
+//                       tau = 0): four partials per request and CTA.
+//   markov_pick_kernel  one CTA per request: merges the partials; at tau > 0
+//                       forms the level-1 key of every 256-entry race block
+//                       from its four sub-blocks, recomputes the winning
+//                       block's 256 logits and draws inside it (level 2);
+//                       writes the draft, its confidence and the row
+//                       statistics, and gathers W1 at the draft into E for
 //                       the next position.
 //
 // Consecutive kernels overlap through programmatic dependent launch: each
@@ -50,18 +51,19 @@ constexpr int kMkTile = 128;        // MMA N: vocabulary rows of W2^T per tile
 constexpr int kMkAtomK = 64;        // bf16 along K per 128-byte swizzle atom
 constexpr int kMkAtomBytes = 128 * 128;  // one atom of 128 rows x 128 bytes
 constexpr int kMkEpiWarps = 8;      // two per TMEM lane quarter, taking alternate tiles
-constexpr int kMkBlock = 64;        // race block of this sampler (two per tile)
+constexpr int kMkSub = 64;          // sub-block: the columns of a tile one epilogue warp takes
+constexpr int kMkRace = kRaceBlock; // race block: four sub-blocks (the blocks of every draw)
 constexpr int kMkThreads = 32 * (2 + kMkEpiWarps);  // warp 0 TMA, warp 1 MMA, then the epilogue
 constexpr int kMkMaxR = 256;
 constexpr int kMkSlots = 4;         // accumulators: tile t in slot t % 4
 constexpr int kMkTmemCols = kMkSlots * kMkTile;  // 512 fp32 columns
-constexpr int kPickThreads = 256;
+constexpr int kPickThreads = 1024;  // level 2: 32 warps x 8 entries = one race block
 
 struct alignas(16) MkPartial {
   float m, s;     // softmax statistics of the CTA's columns (s relative to fl(m*c2))
-  float L;        // tau > 0: best block's log2 E - log2 sum; tau = 0: the max
-  int32_t idx;    // tau > 0: best block; tau = 0: lowest argmax (INT_MAX: none)
-  float M;        // tau > 0: best block's max
+  float L;        // tau = 0: the max
+  int32_t idx;    // tau = 0: lowest argmax (INT_MAX: none)
+  float M;        // unused
   int32_t flags;  // bit0: NaN or +inf
   int32_t pad[2];
 };
@@ -78,6 +80,8 @@ struct MarkovLaunch {
   const int32_t* x0;
   __nv_bfloat16* E;  // [128, r]: W1 at the previous drafts
   MkPartial* part;   // [B][G][4]: per bias CTA, per epilogue half and column half
+  float2* sub;       // [B][nsub_pad]: per 64-column sub-block (max, sum relative to fl(max*c2)), tau > 0
+  int nsub, nsub_pad;
   int G;
   uint32_t* req_bad;  // [B]
   int32_t* drafts;
@@ -349,14 +353,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     const int row = 32 * row_q + lane;
     const bool valid = row < p.B;
     const size_t urow = ((size_t)(valid ? row : 0) * p.K + p.step) * (size_t)p.V;
-    const long long pos = valid ? __ldg(reinterpret_cast<const long long*>(p.pos_base) + row) : 0;
-    const uint32_t position = (uint32_t)(pos + p.step + 1);
-    const uint64_t req = valid ? __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + row) : 0;
-    const uint64_t seed = valid ? __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + row) : 0;
-    const int nblk = dup ? 1 : 2;            // race blocks of a tile this warp takes
+    const int nblk = dup ? 1 : 2;            // sub-blocks of a tile this warp takes
     const int blk0 = dup ? col_half : 0;
     SoftState st{-INFINITY, 0.0f};
-    MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t flags = 0;
     bool aborted = false;
@@ -370,7 +369,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 #pragma unroll
       for (int h = 0; h < 16; ++h) {
         if (h >= 8 * nblk) break;
-        const int v = v0 + kMkBlock * blk0 + 8 * h;
+        const int v = v0 + kMkSub * blk0 + 8 * h;
         if (valid && p.u_vec && v + 8 <= p.V) {
           uw[h] = __ldg(reinterpret_cast<const uint4*>(p.U + urow + v));
         } else {
@@ -384,8 +383,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       }
       // the warp's next tile of U, into L2 while this one is processed
       if (valid && t + 2 < T) {
-        const int vn = ((int)blockIdx.x + (t + 2) * p.G) * kMkTile + kMkBlock * blk0;
-        const int ve = min(vn + kMkBlock * nblk, p.V) - 1;
+        const int vn = ((int)blockIdx.x + (t + 2) * p.G) * kMkTile + kMkSub * blk0;
+        const int ve = min(vn + kMkSub * nblk, p.V) - 1;
         if (vn < p.V)
           for (int x = vn; x <= ve; x += 64) {
             asm volatile("prefetch.global.L2 [%0];" ::"l"(p.U + urow + x));
@@ -399,17 +398,17 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       }
       tc_fence_after();
       for (int cb = 0; cb < nblk; ++cb) {
-        const int bcol = kMkBlock * (blk0 + cb);  // the race block's first column in the tile
-        const int b = (v0 + bcol) / kMkBlock;
+        const int bcol = kMkSub * (blk0 + cb);  // the sub-block's first column in the tile
+        const int sb = (v0 + bcol) / kMkSub;
         SoftState blk{-INFINITY, 0.0f};
 #pragma unroll
-        for (int ch = 0; ch < kMkBlock / 32; ++ch) {
+        for (int ch = 0; ch < kMkSub / 32; ++ch) {
           float l[32];
           tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(slot * kMkTile + bcol + 32 * ch), l);
           float cmax = -INFINITY;
 #pragma unroll
           for (int k = 0; k < 32; ++k) {
-            const uint4& w4 = uw[(kMkBlock * cb + 32 * ch + k) >> 3];
+            const uint4& w4 = uw[(kMkSub * cb + 32 * ch + k) >> 3];
             const int e = k & 7;
             const uint32_t word = e < 2 ? w4.x : e < 4 ? w4.y : e < 6 ? w4.z : w4.w;
             l[k] += (e & 1) ? bf16_hi(word) : bf16_lo(word);  // -inf past V (U reads -inf there, the bias is 0)
@@ -436,16 +435,9 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           }
         }
         if (!valid) continue;
-        // the race block is complete
+        // the sub-block is complete: its statistics for the pick's level 1
         st = mk_merge(st, blk, p.c2);
-        if (!kGreedy && blk.m > -INFINITY && blk.s > 0.0f && blk.s == blk.s) {
-          const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)(b >> 2)), (uint32_t)seed,
-                                  (uint32_t)(seed >> 32));
-          const uint32_t word = (b & 3) == 0 ? rq.x : (b & 3) == 1 ? rq.y : (b & 3) == 2 ? rq.z : rq.w;
-          const float E = -log1pf(-((float)race_m(word) * 0x1p-24f));
-          const MkKey cand{mk_lg2(E) - mk_lg2(blk.s), blk.m, b};
-          if (mk_better(cand, best, p.c2)) best = cand;
-        }
+        if (!kGreedy && sb < p.nsub) p.sub[(size_t)row * p.nsub_pad + sb] = make_float2(blk.m, blk.s);
       }
       // the accumulator is read: the MMA may overwrite it
       tc_fence_before();
@@ -457,9 +449,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       MkPartial o{};
       o.m = st.m;
       o.s = st.s;
-      o.L = kGreedy ? g.v : best.L;
-      o.idx = kGreedy ? g.idx : best.idx;
-      o.M = best.M;
+      o.L = kGreedy ? g.v : 0.0f;
+      o.idx = kGreedy ? g.idx : INT_MAX;
       o.flags = flags;
       MkPartial* dstp = p.part + ((size_t)row * p.G + blockIdx.x) * 4 + 2 * eh;
       dstp[col_half] = o;
@@ -481,72 +472,75 @@ __global__ void __launch_bounds__(kMkThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
-// The draw of one position: merge, level 2, outputs, next E
+// The draw of one position: merge, level 1, level 2, outputs, next E
 // ---------------------------------------------------------------------------
+// MkKey of the best of two candidates, over a warp (xor butterfly).
+__device__ __forceinline__ MkKey mk_warp_best(MkKey k, float c2) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const MkKey ok{__shfl_xor_sync(0xFFFFFFFFu, k.L, o), __shfl_xor_sync(0xFFFFFFFFu, k.M, o),
+                   __shfl_xor_sync(0xFFFFFFFFu, k.idx, o)};
+    if (mk_better(ok, k, c2)) k = ok;
+  }
+  return k;
+}
+
 template <bool kGreedy>
-__global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const MarkovLaunch p) {
+__global__ void __launch_bounds__(kPickThreads, 1) markov_pick_kernel(const MarkovLaunch p) {
+  constexpr int kW = kPickThreads / 32;
   __shared__ __align__(16) __nv_bfloat16 sh_e[kMkMaxR];
-  __shared__ float sh_l[kMkBlock];
-  __shared__ KeyState sh_red[kPickThreads / 32];
-  __shared__ MkPartial sh_part[kPickThreads / 32];
+  __shared__ float sh_l[kMkRace];
+  __shared__ KeyState sh_red[kW];
+  __shared__ MkPartial sh_part[kW];
+  __shared__ MkKey sh_key[kW];
   __shared__ float sh_m, sh_S;
   __shared__ int sh_idx, sh_bad;
   const int i = blockIdx.x;
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   // inputs of the whole draw, read before the wait
   const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
   const uint64_t req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
   const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+  const uint32_t position = (uint32_t)(pos + p.step + 1);
   // the next position's bias kernel may launch now: it prefetches its first
   // W2^T tiles and waits for this grid before it reads E
   pdl_launch_dependents();
   pdl_wait_prerequisites();
-  for (int j = threadIdx.x; j < p.r; j += kPickThreads) sh_e[j] = p.E[(size_t)i * p.r + j];
-  // ---- merge the 4G partials: each thread loads up to four before merging ----
+  if (threadIdx.x < p.r) sh_e[threadIdx.x] = p.E[(size_t)i * p.r + threadIdx.x];
+
+  // ---- tau > 0: this thread's first quad of race blocks (16 sub-blocks),
+  // loaded together with the partials below ----
+  const int nb = (p.V + kMkRace - 1) / kMkRace;  // race blocks
+  const int nq = (nb + 3) / 4;                     // quads (one Philox call each)
+  const float4* subrow = reinterpret_cast<const float4*>(p.sub + (size_t)i * p.nsub_pad);
+  float4 sq[8];
+  if (!kGreedy) {
+    const int q = threadIdx.x;
+#pragma unroll
+    for (int h = 0; h < 8; ++h)
+      sq[h] = q < nq && 16 * q + 2 * h < p.nsub ? __ldcg(subrow + 8 * q + h) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+  }
+
+  // ---- merge the 4G partials of the bias CTAs ----
   {
     SoftState st{-INFINITY, 0.0f};
-    MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
     const int n = 4 * p.G;
     const uint4* src = reinterpret_cast<const uint4*>(p.part + (size_t)i * n);
-    for (int c0 = threadIdx.x; c0 < n; c0 += 4 * kPickThreads) {
-      uint4 lo[4], hi[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int c = c0 + u * kPickThreads;
-        if (c < n) {
-          lo[u] = src[2 * c];
-          hi[u] = src[2 * c + 1];
-        } else {  // an empty partial
-          lo[u] = make_uint4(__float_as_uint(-INFINITY), 0u, __float_as_uint(kGreedy ? -INFINITY : INFINITY),
-                             (uint32_t)INT_MAX);
-          hi[u] = make_uint4(0u, 0u, 0u, 0u);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const float om = __uint_as_float(lo[u].x), os = __uint_as_float(lo[u].y);
-        const float oL = __uint_as_float(lo[u].z), oM = __uint_as_float(hi[u].x);
-        const int oidx = (int)lo[u].w;
-        st = soft_merge(st, SoftState{om, os}, p.c2);
-        f |= (int32_t)hi[u].y;
-        if (kGreedy) {
-          const ArgState a{oL, oidx};
-          if (arg_better(a, g)) g = a;
-        } else {
-          const MkKey k{oL, oM, oidx};
-          if (mk_better(k, best, p.c2)) best = k;
-        }
+    for (int c = threadIdx.x; c < n; c += kPickThreads) {
+      const uint4 lo = __ldcg(src + 2 * c), hi = __ldcg(src + 2 * c + 1);
+      st = soft_merge(st, SoftState{__uint_as_float(lo.x), __uint_as_float(lo.y)}, p.c2);
+      f |= (int32_t)hi.y;
+      if (kGreedy) {
+        const ArgState a{__uint_as_float(lo.z), (int)lo.w};
+        if (arg_better(a, g)) g = a;
       }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       st = soft_merge(st, SoftState{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)},
                       p.c2);
-      const MkKey ok{__shfl_xor_sync(0xFFFFFFFFu, best.L, o), __shfl_xor_sync(0xFFFFFFFFu, best.M, o),
-                     __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
-      if (mk_better(ok, best, p.c2)) best = ok;
       const ArgState og{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
       if (arg_better(og, g)) g = og;
     }
@@ -555,37 +549,70 @@ __global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const Mark
       MkPartial w{};
       w.m = st.m;
       w.s = st.s;
-      w.L = kGreedy ? g.v : best.L;
-      w.idx = kGreedy ? g.idx : best.idx;
-      w.M = best.M;
+      w.L = g.v;
+      w.idx = g.idx;
       w.flags = f;
-      sh_part[threadIdx.x >> 5] = w;
+      sh_part[warp] = w;
     }
+  }
+
+  // ---- level 1 (tau > 0): the key of every 256-entry block from its four
+  // 64-column sub-blocks, log2 E_b - log2 sum_b against the block's max ----
+  if (!kGreedy) {
+    MkKey best{INFINITY, 0.0f, INT_MAX};
+    for (int q = threadIdx.x; q < nq; q += kPickThreads) {
+      if (q != (int)threadIdx.x) {  // quads past the first: loaded here
+#pragma unroll
+        for (int h = 0; h < 8; ++h)
+          sq[h] = 16 * q + 2 * h < p.nsub ? __ldcg(subrow + 8 * q + h) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+      }
+      const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)q), (uint32_t)seed,
+                              (uint32_t)(seed >> 32));
+      const uint32_t words[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+      for (int s4 = 0; s4 < 4; ++s4) {
+        const int b = 4 * q + s4;
+        SoftState blk{-INFINITY, 0.0f};
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const float4 v = sq[2 * s4 + h];
+          // a sub-block past V reads (-inf, 0); a partial sub-block with 16 * q + 2 * h + 1 >= nsub was
+          // loaded whole but its second half is past the row's last sub-block
+          blk = mk_merge(blk, SoftState{v.x, v.y}, p.c2);
+          if (16 * q + 4 * s4 + 2 * h + 1 < p.nsub) blk = mk_merge(blk, SoftState{v.z, v.w}, p.c2);
+        }
+        if (b < nb && blk.m > -INFINITY && blk.s > 0.0f && isfinite(blk.s)) {
+          const float E = -log1pf(-((float)race_m(words[s4]) * 0x1p-24f));
+          const MkKey cand{mk_lg2(E) - mk_lg2(blk.s), blk.m, b};
+          if (mk_better(cand, best, p.c2)) best = cand;
+        }
+      }
+    }
+    best = mk_warp_best(best, p.c2);
+    if (lane == 0) sh_key[warp] = best;
   }
   __syncthreads();
   if (threadIdx.x < 32) {
-    // warp 0 merges the eight warps' results
+    // warp 0 merges the warps' results
     SoftState st{-INFINITY, 0.0f};
     MkKey best{INFINITY, 0.0f, INT_MAX};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    if (lane < kPickThreads / 32) {
+    if (lane < kW) {
       const MkPartial& o = sh_part[lane];
       st = SoftState{o.m, o.s};
       f = o.flags;
-      if (kGreedy) g = ArgState{o.L, o.idx};
-      else best = MkKey{o.L, o.M, o.idx};
+      g = ArgState{o.L, o.idx};
+      if (!kGreedy) best = sh_key[lane];
     }
 #pragma unroll
-    for (int o = (kPickThreads / 32) / 2; o > 0; o >>= 1) {
+    for (int o = kW / 2; o > 0; o >>= 1) {
       st = soft_merge(st, SoftState{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)},
                       p.c2);
-      const MkKey ok{__shfl_xor_sync(0xFFFFFFFFu, best.L, o), __shfl_xor_sync(0xFFFFFFFFu, best.M, o),
-                     __shfl_xor_sync(0xFFFFFFFFu, best.idx, o)};
-      if (mk_better(ok, best, p.c2)) best = ok;
       const ArgState og{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
       if (arg_better(og, g)) g = og;
     }
+    if (!kGreedy) best = mk_warp_best(best, p.c2);
     f = (int32_t)__reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
     if (lane == 0) {
       sh_m = st.m;
@@ -604,23 +631,15 @@ __global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const Mark
     if (kGreedy) {
       z = sh_idx;
     } else {
-      // level 2: the winning block's 64 logits recomputed (U + E . W2^T row).
-      // Warp w takes entries 8w..8w+7 of the block; lane l multiplies the
-      // r-slice 8l..8l+7 of each (one coalesced 16-byte load per entry, all
-      // issued at once), and a transposed butterfly leaves entry 8w + l / 4's
-      // dot product in lanes 4 (l / 4)..4 (l / 4) + 3.
+      // level 2: the winning block's 256 logits recomputed (U + E . W2^T
+      // row).  Warp w takes entries 8w..8w+7 of the block; lane l multiplies
+      // the r-slice 8l..8l+7 of each (one coalesced 16-byte load per entry,
+      // all issued at once), and a transposed butterfly leaves entry
+      // 8w + l / 4's dot product in lanes 4 (l / 4)..4 (l / 4) + 3.
       const int b = sh_idx;
-      const int w_id = threadIdx.x >> 5;
-      const int v_base = b * kMkBlock + 8 * w_id;
+      const int v_base = b * kMkRace + 8 * warp;
       const int v = v_base + (lane >> 2);
       const bool owner = (lane & 3) == 0;
-      // the rows of W1 at the block's entries, into L2: one of them becomes
-      // the next position's E row (thread t: row t / 4, 128-byte line t % 4)
-      if (p.step + 1 < p.K) {
-        const int wv = b * kMkBlock + (threadIdx.x >> 2), line = threadIdx.x & 3;
-        if (wv < p.V && line < p.r / 64)
-          asm volatile("prefetch.global.L2 [%0];" ::"l"(p.W1 + (size_t)wv * p.r + 64 * line));
-      }
       const float u_v = (owner && v < p.V) ? load_elem(p.U + ((size_t)i * p.K + p.step) * (size_t)p.V + v) : 0.0f;
       float part[8];
       {
@@ -665,27 +684,41 @@ __global__ void __launch_bounds__(kPickThreads, 4) markov_pick_kernel(const Mark
       if (owner && v < p.V) {
         l = u_v + part[0];
         const float w = ex2_approx(__fmaf_rn(l, p.c2, -M2));
-        const uint4 rw = philox(draw_counter((uint32_t)(pos + p.step + 1), req, SPEC_PURPOSE_DRAFT_IN_BLOCK,
-                                             (uint32_t)(v >> 2)),
-                                (uint32_t)seed, (uint32_t)(seed >> 32));
+        const uint4 rw =
+            philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT_IN_BLOCK, (uint32_t)(v >> 2)), (uint32_t)seed,
+                   (uint32_t)(seed >> 32));
         const uint32_t word = (v & 3) == 0 ? rw.x : (v & 3) == 1 ? rw.y : (v & 3) == 2 ? rw.z : rw.w;
         if (w > 0.0f) e = KeyState{race_key(race_m(word), w), v};
       }
-      if (owner) sh_l[8 * w_id + (lane >> 2)] = l;
-      e = cta_min_key(e, sh_red);
-      if (threadIdx.x == 0) sh_idx = e.idx == INT_MAX ? -1 : e.idx;
+      if (owner) sh_l[8 * warp + (lane >> 2)] = l;
+      // the lowest key over the CTA
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const KeyState other{__shfl_xor_sync(0xFFFFFFFFu, e.key, o), __shfl_xor_sync(0xFFFFFFFFu, e.idx, o)};
+        if (key_better(other, e)) e = other;
+      }
+      if (lane == 0) sh_red[warp] = e;
+      __syncthreads();
+      if (warp == 0) {
+        KeyState a = lane < kW ? sh_red[lane] : KeyState{INFINITY, INT_MAX};
+#pragma unroll
+        for (int o = kW / 2; o > 0; o >>= 1) {
+          const KeyState other{__shfl_xor_sync(0xFFFFFFFFu, a.key, o), __shfl_xor_sync(0xFFFFFFFFu, a.idx, o)};
+          if (key_better(other, a)) a = other;
+        }
+        if (lane == 0) sh_idx = a.idx == INT_MAX ? -1 : a.idx;
+      }
       __syncthreads();
       z = sh_idx;
-      if (z >= 0) lz = sh_l[z - b * kMkBlock];
+      if (z >= 0) lz = sh_l[z - b * kMkRace];
     }
   }
   // the next position's operand row: W1 at this draft
-  if (p.step + 1 < p.K)
-    for (int j = threadIdx.x; j < p.r; j += kPickThreads) {
-      const __nv_bfloat16 w = p.W1[(size_t)(bad || z < 0 ? 0 : z) * p.r + j];
-      p.E[(size_t)i * p.r + j] = w;
-      if (p.B <= 64) p.E[(size_t)(i + 64) * p.r + j] = w;  // the repeated rows
-    }
+  if (p.step + 1 < p.K && (int)threadIdx.x < p.r) {
+    const __nv_bfloat16 w = p.W1[(size_t)(bad || z < 0 ? 0 : z) * p.r + threadIdx.x];
+    p.E[(size_t)i * p.r + threadIdx.x] = w;
+    if (p.B <= 64) p.E[(size_t)(i + 64) * p.r + threadIdx.x] = w;  // the repeated rows
+  }
   if (threadIdx.x != 0) return;
   const size_t o = (size_t)i * p.K + p.step;
   if (bad || z < 0) {
@@ -772,17 +805,21 @@ static bool make_map(CUtensorMap* map, const void* base, int r, long long rows) 
 }
 
 struct MarkovGeometry {
-  int G;
-  size_t e_off, part_off, bad_off, bytes;
+  int G, nsub, nsub_pad;
+  size_t e_off, part_off, sub_off, bad_off, bytes;
 };
 
 static MarkovGeometry markov_geometry(int B, int V, int r, int sms) {
   MarkovGeometry g{};
   const int ntiles = (V + kMkTile - 1) / kMkTile;
   g.G = std::max(1, std::min(sms, ntiles));
+  // sub-blocks of a row, padded to whole quads of race blocks (16 sub-blocks)
+  g.nsub = (V + kMkSub - 1) / kMkSub;
+  g.nsub_pad = (g.nsub + 15) / 16 * 16;
   g.e_off = 0;
   g.part_off = ((size_t)kMkRows * r * 2 + 255) / 256 * 256;
-  g.bad_off = g.part_off + ((size_t)sizeof(MkPartial) * B * 4 * g.G + 255) / 256 * 256;
+  g.sub_off = g.part_off + ((size_t)sizeof(MkPartial) * B * 4 * g.G + 255) / 256 * 256;
+  g.bad_off = g.sub_off + ((size_t)sizeof(float2) * B * g.nsub_pad + 255) / 256 * 256;
   g.bytes = g.bad_off + ((size_t)4 * B + 255) / 256 * 256;
   return g;
 }
@@ -842,6 +879,9 @@ extern "C" int spec_markov_draft(const void* U, int u_dtype, const void* W1, con
   char* base = static_cast<char*>(ws);
   p.E = reinterpret_cast<__nv_bfloat16*>(base + g.e_off);
   p.part = reinterpret_cast<MkPartial*>(base + g.part_off);
+  p.sub = reinterpret_cast<float2*>(base + g.sub_off);
+  p.nsub = g.nsub;
+  p.nsub_pad = g.nsub_pad;
   p.G = g.G;
   p.req_bad = reinterpret_cast<uint32_t*>(base + g.bad_off);
   p.drafts = drafts_out;

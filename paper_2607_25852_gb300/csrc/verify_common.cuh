@@ -364,7 +364,8 @@ struct Row8<float> {
 // Philox work is 1/kRaceBlock of a per-entry race, and level 2 touches one
 // block.  Block variates use purpose SAMPLE (sub-index b / 4, word b % 4), entry
 // variates purpose SAMPLE_IN_BLOCK (sub-index v / 4, word v % 4).
-constexpr int kRaceBlock = 256;              // entries per block (one warp step: 32 lanes x 8)
+constexpr int kRaceBlock = SPEC_RACE_BLOCK;  // entries per block (one warp step here: 32 lanes x 8)
+static_assert(kRaceBlock == 256, "the race kernels take a block as one warp step of 32 lanes x 8 entries");
 constexpr int kRaceQuad = 4 * kRaceBlock;    // the four blocks of one Philox call
 
 // Race variate of a Philox word: E = -ln(u), u = (2 * (word >> 9) + 1) * 2^-24.

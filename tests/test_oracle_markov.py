@@ -32,35 +32,30 @@ def _case(B, K, V, r, seed, std=2.0, wstd=0.3):
     return U, bf16_bits_from_float(W1), bf16_bits_from_float(W2), _bf16(W1), _bf16(W2), x0, seeds, rids, pos
 
 
-@pytest.mark.parametrize("tau", [0.0, 0.8])
+@pytest.mark.parametrize("tau", [0.0, 0.8, 1.0])
 def test_zero_transition_is_the_draft_step(tau):
-    """W1 = 0: every bias vanishes, so each position's q is the draft step's.
-    The row statistics agree exactly; at tau = 0 so do the drafts.  At
-    tau > 0 the two races block the vocabulary differently (64 against 256
-    entries; each is an exact draw), so each confidence is checked as q at
-    the Markov draw."""
-    U, _, _, _, _, x0, seeds, rids, pos = _case(3, 5, 600, 8, 1)
-    zero1 = np.zeros((600, 8), np.uint16)
-    zero2 = np.zeros((8, 600), np.uint16)
+    """W1 = 0: every bias vanishes, so each position's q is the draft step's,
+    and both draws race the same 256-entry blocks with the same variates
+    (purposes DRAFT and DRAFT_IN_BLOCK at the drafted position): drafts,
+    confidences, scores and row statistics all agree exactly, at tau = 0 and
+    tau > 0.  V = 1100 puts the winner in any of five blocks, the last one
+    partial."""
+    U, _, _, _, _, x0, seeds, rids, pos = _case(16, 5, 1100, 8, 1)
+    zero1 = np.zeros((1100, 8), np.uint16)
+    zero2 = np.zeros((8, 1100), np.uint16)
     mk = oracle.markov_batch(U, zero1, zero2, x0, tau, seeds, rids, pos)
     dr = oracle.draft_batch(U, tau, seeds, rids, pos)
-    for k in ("m", "logS", "status"):
+    for k in ("z", "c", "s", "m", "logS", "status"):
         assert np.array_equal(mk[k], dr[k]), k
-    if tau == 0:
-        for k in ("z", "c", "s"):
-            assert np.array_equal(mk[k], dr[k]), k
-    tc = tau if tau > 0 else 1.0                  # confidences at temperature 1 when greedy
-    q = np.exp(U.astype(np.float64) / tc - mk["m"][..., None] - mk["logS"][..., None])
-    for i in range(3):
-        for k in range(5):
-            assert mk["c"][i, k] == pytest.approx(q[i, k, mk["z"][i, k]], rel=1e-12)
+    if tau > 0:
+        assert len(set((mk["z"] // 256).ravel().tolist())) >= 3    # the draws span several blocks
 
 
-def test_race_blocks_of_64_follow_q():
-    """The Markov draw races blocks of 64 entries: V = 300 (five blocks, the
-    last one partial), 20000 requests with zero bias, the draft's histogram
-    over the blocks against q's block masses (chi-square, 4 dof)."""
-    V, N = 300, 20000
+def test_race_blocks_follow_q():
+    """The Markov draw's level-1 blocks hold 256 entries: V = 1100 (five
+    blocks, the last partial), 20000 requests with zero bias, the draft's
+    histogram over the blocks against q's block masses (chi-square, 4 dof)."""
+    V, N = 1100, 20000
     rng = np.random.default_rng(11)
     row = rng.normal(0, 1.0, V).astype(np.float32)
     U = np.broadcast_to(row, (N, 1, V)).copy()
@@ -68,8 +63,8 @@ def test_race_blocks_of_64_follow_q():
                               1.0, np.full(N, 3, np.uint64), np.arange(N, dtype=np.uint64), np.full(N, 9, np.int64))
     q = np.exp(row.astype(np.float64) - row.max())
     q /= q.sum()
-    mass = np.array([q[b * 64:(b + 1) * 64].sum() for b in range(5)])
-    counts = np.bincount(res["z"][:, 0] // 64, minlength=5)
+    mass = np.array([q[b * 256:(b + 1) * 256].sum() for b in range(5)])
+    counts = np.bincount(res["z"][:, 0] // 256, minlength=5)
     chi2 = ((counts - N * mass) ** 2 / (N * mass)).sum()
     assert stats.chi2.sf(chi2, 4) > 1e-3
 
