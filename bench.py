@@ -39,7 +39,7 @@ sys.path.insert(0, ROOT)
 METRIC = "verified positions/s"
 UNIT = "positions/s"
 L2_BYTES = 129 * 1000 * 1000  # GB300 L2, 129 MB
-PROFILE_EVERY = 8  # steps between two timings of the streaming kernel
+KERNEL_SAMPLES = 30  # event-bracketed launches of the streaming kernel, at least
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -283,9 +283,30 @@ def recorded_traffic(workload):
 # ---------------------------------------------------------------------------
 # CPU oracle timings (test infrastructure, timed as a reported baseline)
 # ---------------------------------------------------------------------------
-def oracle_sample(wl, seconds, step_repeats=None):
-    """Run the CPU oracle over full batches of the same workload on all host
-    cores (one request per task) until `seconds` of wall time have passed."""
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else platform)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def oracle_sample(wl, seconds, step_repeats=None, max_threads=None):
+    """Run the CPU oracle over full batches of the same workload on the host
+    cores (one request per task; at most `max_threads` threads) until
+    `seconds` of wall time have passed."""
     import oracle
     import torch
     lg = wl.logits.detach().cpu()
@@ -308,6 +329,8 @@ def oracle_sample(wl, seconds, step_repeats=None):
     rows = 0
     batches = 0
     t0 = time.perf_counter()
+    if max_threads is not None:
+        threads = max(1, min(threads, max_threads))
     with cf.ThreadPoolExecutor(max_workers=threads) as ex:
         while True:
             list(ex.map(one, range(B)))
@@ -384,9 +407,7 @@ def run_ours(args):
     # ---- device-timed region ----
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
-    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
-    for pair in ev + kev:          # torch creates the CUDA events lazily, at first record
+    for pair in ev:                # torch creates the CUDA events lazily, at first record
         for e in pair:
             e.record(stream)
     # A step whose inputs fit in L2 would find them cached from the step
@@ -405,11 +426,6 @@ def run_ours(args):
             if flush is not None:
                 flush.fill_(k & 0xFF)
             ev[k][0].record(stream)
-            if k % PROFILE_EVERY == 0:
-                # events around the streaming kernel of every PROFILE_EVERY-th
-                # step: an event between two kernels breaks their programmatic
-                # overlap, so the other steps run without them
-                spec.spec_profile_stream_pass(kev[k][0], kev[k][1])
             step.run()
             ev[k][1].record(stream)
         stop.record(stream)
@@ -420,9 +436,27 @@ def run_ours(args):
         total_ms = sum(a.elapsed_time(b) for a, b in ev)
     total_ms = max_over_ranks(dist, total_ms, device)
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    kern_ms = [kev[k][0].elapsed_time(kev[k][1]) for k in range(0, args.steps, PROFILE_EVERY)]
     ms_per_step = total_ms / args.steps
     value = job_throughput(world, R, args.steps, total_ms)
+
+    # ---- the streaming kernel alone: its own loop of event-bracketed steps ----
+    # Events between two kernels break their programmatic overlap, so they
+    # stay out of the timed steps above; here every step brackets the
+    # streaming kernel, and the clocks are sampled over this loop.
+    n_k = max(KERNEL_SAMPLES, args.steps)
+    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_k)]
+    for pair in kev:
+        for e in pair:
+            e.record(stream)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as kclocks:
+        for k in range(n_k):
+            if flush is not None:
+                flush.fill_(k & 0xFF)
+            spec.spec_profile_stream_pass(kev[k][0], kev[k][1])
+            step.run()
+        torch.cuda.synchronize()
+    kern_ms = [a.elapsed_time(b) for a, b in kev]
 
     # ---- the same step captured once in a CUDA graph and replayed ----
     graph = None
@@ -523,21 +557,29 @@ def run_ours(args):
         return 0
 
     peak, peak_kind = measured_peak()
-    k_ms = statistics.mean(kern_ms)
-    achieved = alg["logits"] / (k_ms * 1e-3) / 1e9
+    k_med = statistics.median(kern_ms)
+    achieved = alg["logits"] / (k_med * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
                 "kernel": "stream_rows_kernel", "peak_kind": peak_kind,
-                "algorithmic_bytes_per_launch": alg["logits"], "avg_launch_us": round(1e3 * k_ms, 2),
+                "algorithmic_bytes_per_launch": alg["logits"],
+                "median_launch_us": round(1e3 * k_med, 2),
+                "avg_launch_us": round(1e3 * statistics.mean(kern_ms), 2),
+                "launch_us_p10_p90": [round(1e3 * float(np.percentile(kern_ms, q)), 2) for q in (10, 90)],
+                "launches_timed": len(kern_ms), "clocks": kclocks.summary(),
                 "frac_of_8000": round(achieved / 8000.0, 4)}
     step_gbs = alg["total"] / (ms_per_step * 1e-3) / 1e9
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         rows, el, threads, batches = oracle_sample(wl, args.cpu_seconds)
+        rows1, el1, _, batches1 = oracle_sample(wl, args.cpu_seconds, max_threads=1)
         cpu = {"value": rows / el, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"{batches} full batch(es) of the same workload ({wl.B} requests x "
-                         f"{wl.K + 1} rows), {el:.1f} s wall on {threads} host threads"}
+                         f"{wl.K + 1} rows), {el:.1f} s wall on {threads} host threads",
+               "single_thread": {"value": rows1 / el1, "unit": UNIT, "cores": 1,
+                                 "sample": f"{batches1} full batch(es), {el1:.1f} s wall on 1 thread"},
+               "nproc": os.cpu_count(), "cpu_model": cpu_model()}
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
