@@ -321,28 +321,48 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
   __syncthreads();
 
   // ---- Eq. (dcut-score): fp32 prefix products, request i in thread i ----
+  // Each request's keys go to a run of KP = next power of two >= K slots,
+  // padded with key 0 (below every real key), in descending order for even i
+  // and ascending order for odd i when B * KP <= 1024: the runs are then the
+  // sorted, alternating blocks that the bitonic network's first log2(KP)
+  // levels would produce, and those levels are skipped.
+  const int KP = K <= 1 ? 1 : 1 << (32 - __clz(K - 1));
+  const bool runs = B * KP <= kSmallSlots;
   if (tid < B) {
     const float* ci = sh_conf + tid * CS;
     float s = 1.0f;
-    for (int k = 1; k <= K; ++k) {
-      float c = ci[k - 1];
-      if (!(c >= 0.0f && c <= 1.0f)) {
-        sh_bad = 1;
-        c = 0.0f;
+    for (int k0 = 1; k0 <= K; k0 += 4) {
+      float c4[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) c4[u] = k0 + u <= K ? ci[k0 + u - 1] : 1.0f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k = k0 + u;
+        if (k > K) break;
+        float c = c4[u];
+        if (!(c >= 0.0f && c <= 1.0f)) {
+          sh_bad = 1;
+          c = 0.0f;
+        }
+        c = __fadd_rn(c, 0.0f);  // -0 counts as +0 (its sign bit would break the key order)
+        s = __fmul_rn(s, c);
+        const int slot = runs ? tid * KP + ((tid & 1) ? KP - k : k - 1) : tid * K + (k - 1);
+        sh_x[0][slot] = position_key(s, k, tid);
       }
-      c = __fadd_rn(c, 0.0f);  // -0 counts as +0 (its sign bit would break the key order)
-      s = __fmul_rn(s, c);
-      sh_x[0][tid * K + (k - 1)] = position_key(s, k, tid);
     }
+    if (runs)
+      for (int k = K + 1; k <= KP; ++k) sh_x[0][tid * KP + ((tid & 1) ? KP - k : k - 1)] = 0ull;
   }
   __syncthreads();
 
   // ---- bitonic sort of the draft keys, descending ----
-  unsigned long long x = tid < NK ? sh_x[0][tid] : 0ull;
+  const int NS = runs ? B * KP : NK;  // occupied slots
+  unsigned long long x = tid < NS ? sh_x[0][tid] : 0ull;
   int buf = 1;
-#pragma unroll 1
+#pragma unroll
   for (int k = 2; k <= kSmallSlots; k <<= 1) {
-#pragma unroll 1
+    if (runs && k <= KP) continue;  // the runs are sorted blocks of KP already
+#pragma unroll
     for (int j = k >> 1; j > 0; j >>= 1) {
       unsigned long long y;
       if (j >= 32) {
