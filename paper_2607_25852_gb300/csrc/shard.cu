@@ -360,7 +360,7 @@ __global__ void __launch_bounds__(32) shard_decide_kernel(const ShardLaunch p) {
   }
   bad = __any_sync(0xFFFFFFFFu, bad);
   __syncwarp();
-  decide_chain<kGreedy>(p, i, rs, pre, DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}, lz, qz, bad);
+  decide_chain<kGreedy>(p, i, rs, pre, DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}, lz, qz, bad, true, p.req_rec + i);
 }
 
 // ---------------------------------------------------------------------------

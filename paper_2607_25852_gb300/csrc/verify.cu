@@ -77,7 +77,8 @@ VerifyGeometry verify_geometry(int B, int K, int V) {
 // decision chain.  Only one warp of a CTA decides at a time (its shared arrays
 // are per CTA).
 template <typename T, bool kGreedy>
-__device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre) {
+__device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre,
+                                            bool outputs, ReqRec* rec_dst) {
   const int K = p.K, V = p.V, NC = p.NC;
   const float c2 = p.c2;
   const int lane = threadIdx.x & 31;
@@ -162,14 +163,17 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
     if (sh_z[j] < 0 || sh_z[j] >= V) bad = 1;
   bad = __any_sync(0xFFFFFFFFu, bad);
   __syncwarp();
-  decide_chain<kGreedy>(p, i, rs, pre, DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}, lz, qz, bad);
-  if (lane == 0) p.req_count[i] = 0u;  // leave the workspace zeroed for the next call
+  decide_chain<kGreedy>(p, i, rs, pre, DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}, lz, qz, bad, outputs, rec_dst);
+  if (kGreedy && lane == 0) p.req_count[i] = 0u;  // leave the workspace zeroed for the next call
   __syncwarp();
 }
 
 // End of one (request, row, chunk) item, all threads of the CTA: the CTA
-// reduction and the chunk partial (valid requests), the arrival on the
-// request's counter, and the request's decision if this CTA arrived last.
+// reduction and the chunk partial (valid requests).  At t = 0 the CTA then
+// arrives on the request's counter, and the last CTA to arrive decides the
+// request.  At t > 0 the sampling kernel, which waits for this grid anyway,
+// decides each request from the complete partials, so a streaming CTA ends
+// with its partial and holds no SM slot for a round trip.
 template <typename T, bool kGreedy>
 __device__ __forceinline__ void finish_item(const VerifyLaunch& p, RowAcc<T, kGreedy>& acc, int i, const ReqShape& rs,
                                             long long r, int c) {
@@ -178,6 +182,7 @@ __device__ __forceinline__ void finish_item(const VerifyLaunch& p, RowAcc<T, kGr
     const RowPartial out = cta_reduce_partial<T, kGreedy>(acc, p.c2);
     if (threadIdx.x == 0) p.row_part[(size_t)r * p.NC + c] = out;
   }
+  if (!kGreedy) return;
   // ---- arrival; the last CTA of the request decides it (warp 0) ----
   DecidePre pre;
   if (threadIdx.x < 32) pre = decide_prefetch(p, i);
@@ -189,7 +194,7 @@ __device__ __forceinline__ void finish_item(const VerifyLaunch& p, RowAcc<T, kGr
   consumer_sync();
   if (!sh_last || threadIdx.x >= 32) return;
   __threadfence();  // the other CTAs' partials after their counts
-  decide_request<T, kGreedy>(p, i, rs, pre);
+  decide_request<T, kGreedy>(p, i, rs, pre, true, nullptr);
 }
 
 // Item of CTA blockIdx.x: (request i, row j, chunk c), request-major, so
@@ -236,13 +241,17 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   const int cs = blockIdx.x - i * p.NCS;
   const int V = p.V;
   const int warp = threadIdx.x >> 5;
-  pdl_wait_prerequisites();  // the decisions of the streaming kernel
+  __shared__ ReqRec sh_rec;
+  pdl_wait_prerequisites();  // the row partials of the streaming kernel
   pdl_launch_dependents();   // the commit kernel waits for this grid in turn
-  const ReqRec rec = p.req_rec[i];
+  // The request's decision chain (every CTA of the request runs it, chunk 0
+  // writes the outputs): which row to sample, and how.
+  if (warp == 0) decide_request<T, false>(p, i, request_shape(p, i), decide_prefetch(p, i), cs == 0, &sh_rec);
+  __syncthreads();
+  const ReqRec rec = sh_rec;
   if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
-  // The record comes from this call's decision when the workspace started
-  // zeroed; refuse one that could not (e.g. a workspace the caller did not
-  // leave as the library left it) rather than read outside the inputs.
+  // A record that could not come from a consistent decision is refused
+  // rather than used to read outside the inputs.
   if (rec.a < 0 || rec.a > p.K || rec.srow < 0 || rec.srow >= p.R_max || rec.z_excl < -1 || rec.z_excl >= V ||
       ((rec.flags & 4) && (p.q == nullptr || rec.a >= p.K))) {
     if (threadIdx.x == 0) report(p.status, SPEC_ERR_WORKSPACE);

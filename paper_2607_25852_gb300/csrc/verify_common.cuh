@@ -677,10 +677,14 @@ struct DecideArrays {
   float* pz;
 };
 
+// `outputs`: write the request's outputs (several CTAs may run the same
+// decision; one of them writes); `rec_dst` (t > 0): where the record of the
+// row to sample goes.
 template <bool kGreedy, class L>
 __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& rs, const DecidePre& pre,
                                              const DecideArrays& sh, const float (&lz)[(kMaxRows + 31) / 32],
-                                             const float (&qz)[(kMaxRows + 31) / 32], int bad) {
+                                             const float (&qz)[(kMaxRows + 31) / 32], int bad, bool outputs,
+                                             ReqRec* rec_dst) {
   const int K = p.K;
   const float c2 = p.c2;
   const int lane = threadIdx.x & 31;
@@ -729,7 +733,9 @@ __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& 
 
   const int a = bad ? 0 : first_reject;
   int32_t* tok = p.out_tokens + (size_t)i * (K + 1);
-  if (bad) {
+  if (!outputs) {
+    // another CTA writes this request's outputs
+  } else if (bad) {
     if (lane == 0) report(p.status, SPEC_ERR_BAD_INPUT);
     for (int j = lane; j <= K; j += 32) tok[j] = -1;
     if (lane == 0) p.accepted_len[i] = 0;
@@ -760,7 +766,7 @@ __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& 
   }
   if (lane == 0) {
     if (kGreedy) {
-      if (!bad) tok[a] = sh_g[a];
+      if (!bad && outputs) tok[a] = sh_g[a];
     } else {
       ReqRec rec;
       rec.a = a;
@@ -770,7 +776,7 @@ __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& 
       rec.srow = row0 + a;
       rec.M2 = bad ? 0.0f : sh_m[a] * c2;
       rec.invS = bad ? 0.0f : 1.0f / sh_S[a];
-      p.req_rec[i] = rec;
+      *rec_dst = rec;
     }
   }
   __syncwarp();
