@@ -189,7 +189,7 @@ int spec::verify_impl(const void* logits, int logits_dtype, const int32_t* row_o
   char* base = static_cast<char*>(ws);
   p.row_part = reinterpret_cast<spec::RowPartial*>(base + g.row_part_off);
   p.race_part = reinterpret_cast<spec::RacePartial*>(base + g.race_part_off);
-  p.req_rec = reinterpret_cast<spec::ReqRec*>(base + g.req_rec_off);
+  p.draft_view = reinterpret_cast<float2*>(base + g.view_off);
   p.counters = reinterpret_cast<uint32_t*>(base + g.counters_off);
   p.req_count = p.counters + B;
   p.R_max = B * (K + 1);

@@ -185,7 +185,7 @@ struct VerifyLaunch {
   // workspace carve-up
   RowPartial* row_part;   // [R_max * NC]
   RacePartial* race_part; // [B * NCS]
-  ReqRec* req_rec;        // [B]
+  float2* draft_view;     // [R_max]: (logit, q) at each row's draft token (t > 0)
   uint32_t* counters;     // [B] sampling-pass arrivals per request
   uint32_t* req_count;    // [B] streaming-pass arrivals per request
   int R_max;              // B * (K + 1)
@@ -230,7 +230,7 @@ struct CommitLaunch {
 // Workspace geometry (device independent).
 struct VerifyGeometry {
   int NC, chunk, NCS, chunk_s;
-  size_t row_part_off, race_part_off, req_rec_off, counters_off, bytes;  // [counters_off, bytes) starts at zero
+  size_t row_part_off, race_part_off, view_off, counters_off, bytes;  // [counters_off, bytes) starts at zero
 };
 VerifyGeometry verify_geometry(int B, int K, int V);
 

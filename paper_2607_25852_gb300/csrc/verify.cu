@@ -62,9 +62,9 @@ VerifyGeometry verify_geometry(int B, int K, int V) {
   g.chunk_s = (int)chunk_s;
   g.row_part_off = 0;
   g.race_part_off = round_up((long long)sizeof(RowPartial) * R_max * nc, 256);
-  g.req_rec_off = g.race_part_off + round_up((long long)sizeof(RacePartial) * B * ncs, 256);
+  g.view_off = g.race_part_off + round_up((long long)sizeof(RacePartial) * B * ncs, 256);
   // zero region: sampling arrivals [B], then streaming arrivals [B]
-  g.counters_off = g.req_rec_off + round_up((long long)sizeof(ReqRec) * B, 256);
+  g.counters_off = g.view_off + round_up((long long)sizeof(float2) * R_max, 256);
   g.bytes = g.counters_off + round_up(sizeof(uint32_t) * 2LL * B, 256);
   return g;
 }
@@ -90,15 +90,22 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
   const int n = rs.n;
   const long long row0 = rs.row0;
 
-  // ---- draft tokens (prefetched) ----
-#pragma unroll
-  for (int u = 0; u < (kMaxRows + 31) / 32; ++u)
-    if (lane + 32 * u < K) sh_z[lane + 32 * u] = pre.z[u];
-  __syncwarp();
-
-  // ---- round trip 2: row partials (a lane per row) and, per draft, the
-  // target logit and the draft probability at the drafted token ----
+  // ---- one round trip: the row partials (a lane per row), at t > 0 each
+  // row's (target logit, q) at its draft from the streaming pass, and the
+  // draft tokens (prefetched by the caller) ----
   int bad = rs.valid ? 0 : 1;
+  float lz[(kMaxRows + 31) / 32], qz[(kMaxRows + 31) / 32];
+#pragma unroll
+  for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
+    const int j = lane + 32 * u;
+    lz[u] = 0.0f;
+    qz[u] = 1.0f;
+    if (!kGreedy && rs.valid && j < n) {
+      const float2 v = __ldcg(p.draft_view + row0 + j);
+      lz[u] = v.x;
+      qz[u] = v.y;
+    }
+  }
   if (rs.valid) {
     for (int j = lane; j <= n; j += 32) {
       const RowPartial* part = p.row_part + (size_t)(row0 + j) * NC;
@@ -143,22 +150,10 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
       }
     }
   }
-  float lz[(kMaxRows + 31) / 32], qz[(kMaxRows + 31) / 32];
-  if (!kGreedy && rs.valid) {
 #pragma unroll
-    for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
-      const int j = lane + 32 * u;
-      lz[u] = 0.0f;
-      qz[u] = 1.0f;
-      if (j < n) {
-        const int z = sh_z[j];
-        if (z >= 0 && z < V) {
-          lz[u] = load_elem(static_cast<const T*>(p.logits) + (size_t)(row0 + j) * V + z);
-          if (p.q) qz[u] = load_any(p.q, p.q_dtype, ((int64_t)i * K + j) * (int64_t)V + z);
-        }
-      }
-    }
-  }
+  for (int u = 0; u < (kMaxRows + 31) / 32; ++u)
+    if (lane + 32 * u < K) sh_z[lane + 32 * u] = pre.z[u];
+  __syncwarp();
   for (int j = lane; j < n; j += 32)
     if (sh_z[j] < 0 || sh_z[j] >= V) bad = 1;
   bad = __any_sync(0xFFFFFFFFu, bad);
@@ -228,7 +223,18 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
   if (rs.valid) {
     const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.V;
     const int v0 = it.c * p.chunk;
-    stream_chunk<T, kGreedy>(acc, row, v0, min(p.V, v0 + p.chunk), 0, p.c2);
+    const int v1 = min(p.V, v0 + p.chunk);
+    // t > 0: the row's draft token, loaded while the chunk streams; the CTA
+    // whose chunk holds it records the target logit and q there for the
+    // decision (a draft outside [0, V) is left to the decision to report)
+    int z = -1;
+    if (!kGreedy && threadIdx.x == 0 && it.j < rs.n) z = __ldg(p.drafts + (size_t)it.i * p.K + it.j);
+    stream_chunk<T, kGreedy>(acc, row, v0, v1, 0, p.c2);
+    if (!kGreedy && threadIdx.x == 0 && z >= v0 && z < v1) {
+      const float lz = load_elem(row + z);
+      const float qz = p.q ? load_any(p.q, p.q_dtype, ((int64_t)it.i * p.K + it.j) * (int64_t)p.V + z) : 1.0f;
+      p.draft_view[r] = make_float2(lz, qz);
+    }
   }
   finish_item<T, kGreedy>(p, acc, it.i, rs, r, it.c);
 }
