@@ -286,6 +286,15 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
 // ends request i's kept prefix.
 constexpr int kSmallSlots = kAllocThreads;
 
+// units * 2^-40 as a double, for 0 < units < 2^53 (exact), with integer
+// operations only: the product's exponent and mantissa fields are set directly.
+__device__ __forceinline__ double units_to_double(long long units) {
+  const int msb = 63 - __clzll(units);
+  const unsigned long long mant = ((unsigned long long)units << (63 - msb)) << 1 >> 12;  // the bits below the msb
+  const unsigned long long expo = (unsigned long long)(msb - 40 + 1023);
+  return __longlong_as_double((long long)((expo << 52) | mant));
+}
+
 __device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long x, int o) {
   const unsigned lo = __shfl_xor_sync(0xFFFFFFFFu, (unsigned)x, o);
   const unsigned hi = __shfl_xor_sync(0xFFFFFFFFu, (unsigned)(x >> 32), o);
@@ -328,6 +337,11 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
   // levels would produce, and those levels are skipped.
   const int KP = K <= 1 ? 1 : 1 << (32 - __clz(K - 1));
   const bool runs = B * KP <= kSmallSlots;
+  // Keys are staged with a row of RL slots per request at the odd stride
+  // RS = RL + 1 (in 8-byte words), so that the threads of a half-warp, one
+  // request each, store to distinct banks.
+  const int RL = runs ? KP : (K > 0 ? K : 1), RS = RL + 1;
+  unsigned long long* stage = &sh_x[0][0];  // B * RS <= 2048 words over both buffers
   if (tid < B) {
     const float* ci = sh_conf + tid * CS;
     float s = 1.0f;
@@ -346,18 +360,19 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
         }
         c = __fadd_rn(c, 0.0f);  // -0 counts as +0 (its sign bit would break the key order)
         s = __fmul_rn(s, c);
-        const int slot = runs ? tid * KP + ((tid & 1) ? KP - k : k - 1) : tid * K + (k - 1);
-        sh_x[0][slot] = position_key(s, k, tid);
+        const int slot = tid * RS + (runs && (tid & 1) ? KP - k : k - 1);
+        stage[slot] = position_key(s, k, tid);
       }
     }
     if (runs)
-      for (int k = K + 1; k <= KP; ++k) sh_x[0][tid * KP + ((tid & 1) ? KP - k : k - 1)] = 0ull;
+      for (int k = K + 1; k <= KP; ++k) stage[tid * RS + ((tid & 1) ? KP - k : k - 1)] = 0ull;
   }
   __syncthreads();
 
   // ---- bitonic sort of the draft keys, descending ----
   const int NS = runs ? B * KP : NK;  // occupied slots
-  unsigned long long x = tid < NS ? sh_x[0][tid] : 0ull;
+  unsigned long long x = tid < NS ? stage[(tid / RL) * RS + tid % RL] : 0ull;
+  __syncthreads();  // the staging area is the exchange buffer from here on
   int buf = 1;
 #pragma unroll
   for (int k = 2; k <= kSmallSlots; k <<= 1) {
@@ -393,25 +408,27 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
 
   // ---- Eq. (dcut-select): first maximiser of U / cost ----
   if (tid < 32) {
-    double best_obj = -INFINITY;
+    long long best_key = -1;
     int best_c = INT_MAX;
     for (int c = tid; c < p.M; c += 32) {
       const int td = p.cand_T[c] - B;  // draft positions kept at this budget
       const long long Uq = ((long long)B << 40) + (td > 0 ? prefix[td - 1] : 0);
-      const double U = (double)Uq * 0x1p-40;
+      const double U = units_to_double(Uq);
       if (p.utility_out) p.utility_out[c] = U;
-      const double obj = U / p.cand_cost[c];
-      if (obj > best_obj) {  // c increases along the lane's loop
-        best_obj = obj;
+      // U > 0 and cost > 0: the bit patterns of the quotients order as the
+      // quotients do, so the comparisons below are integer ones
+      const long long obj = __double_as_longlong(U / p.cand_cost[c]);
+      if (obj > best_key) {  // c increases along the lane's loop
+        best_key = obj;
         best_c = c;
       }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-      const double ob = __shfl_xor_sync(0xFFFFFFFFu, best_obj, o);
+      const long long ob = __shfl_xor_sync(0xFFFFFFFFu, best_key, o);
       const int cb = __shfl_xor_sync(0xFFFFFFFFu, best_c, o);
-      if (ob > best_obj || (ob == best_obj && cb < best_c)) {
-        best_obj = ob;
+      if (ob > best_key || (ob == best_key && cb < best_c)) {
+        best_key = ob;
         best_c = cb;
       }
     }
