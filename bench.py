@@ -195,8 +195,16 @@ class Step:
         self.spec = spec
         self.wl = wl
         B, K, V = wl.B, wl.K, wl.V
-        self.ratios = spec.spec_budget_from_ratios(B, K, [1, 1, 3, 1], [4, 2, 4, 1])
-        self.costs = [1.0, 1.0, 1.0, 1.0]
+        if wl.name == "alloc":
+            # the alloc workload's budget sweep T = 64..1024 with the profiled
+            # piecewise-linear cost: D-cut picks T* < B(K+1)
+            import workloads
+            Ts, costs = workloads.budget_candidates(B, K)
+            self.ratios, self.costs = [int(t) for t in Ts], [float(c) for c in costs]
+        else:
+            # the paper's ratios 1/4..1 with a flat cost table: the full block wins
+            self.ratios = spec.spec_budget_from_ratios(B, K, [1, 1, 3, 1], [4, 2, 4, 1])
+            self.costs = [1.0, 1.0, 1.0, 1.0]
         i32, i64 = torch.int32, torch.int64
         z = lambda *s, dt=i32: torch.zeros(s, dtype=dt, device=device)
         self.depth, self.row_off = z(B), z(B + 1)
@@ -208,12 +216,25 @@ class Step:
         self.hout = None if wl.hidden is None else torch.empty_like(wl.hidden)
         self.status = z(1)
         self.ws = spec.verify_workspace(B, K, V, device)
+        # The target forward writes its rows in the packed order of the
+        # allocation; it is not part of this library, so the packed logits
+        # and hidden rows of the (fixed) allocation are prepared once here.
+        self.logits, self.hidden = wl.logits, wl.hidden
+        spec.spec_allocate(wl.conf, self.ratios, self.costs, wl.last_tokens, wl.drafts, wl.pos_base,
+                           self.depth, self.row_off, self.ptok, self.ppos, self.chosen, self.util, self.status)
+        torch.cuda.synchronize()
+        self.rows = int(self.chosen.item())
+        if self.rows < wl.rows:
+            import workloads
+            depth = self.depth.cpu()
+            self.logits = workloads.pack_rows(wl.logits, B, K, depth)
+            self.hidden = None if wl.hidden is None else workloads.pack_rows(wl.hidden, B, K, depth)
 
     def run(self, inputs=None):
         wl = self.wl
-        x = inputs or dict(conf=wl.conf, logits=wl.logits, drafts=wl.drafts, q=wl.q, seeds=wl.seeds,
+        x = inputs or dict(conf=wl.conf, logits=self.logits, drafts=wl.drafts, q=wl.q, seeds=wl.seeds,
                            request_ids=wl.request_ids, pos_base=wl.pos_base,
-                           last_tokens=wl.last_tokens, hidden=wl.hidden)
+                           last_tokens=wl.last_tokens, hidden=self.hidden)
         s = self.spec
         s.spec_allocate(x["conf"], self.ratios, self.costs, x["last_tokens"], x["drafts"],
                         x["pos_base"], self.depth, self.row_off, self.ptok, self.ppos, self.chosen,
@@ -230,14 +251,15 @@ class Step:
         return 1 + (1 if self.wl.temperature == 0 else 2) + (1 if self.wl.B <= 256 else 2)
 
 
-def algorithmic_bytes(wl, acc):
+def algorithmic_bytes(wl, acc, rows=None):
     """Bytes the method must move once per step (Section 4.2 verifies every
-    retained position in one pass): every logits row, the q row at each
-    rejection, the q(z)/l(z) gathers, the committed hidden rows read and
-    written, and the small per-request arrays."""
+    retained position in one pass): every kept logits row (`rows`, all
+    B(K+1) by default), the q row at each rejection, the q(z)/l(z) gathers,
+    the committed hidden rows read and written, and the small per-request
+    arrays."""
     B, K, V, H = wl.B, wl.K, wl.V, wl.H
     esize = 2 if wl.dtype == "bf16" else 4
-    logits = B * (K + 1) * V * esize
+    logits = (B * (K + 1) if rows is None else rows) * V * esize
     rejected = int(np.sum(acc < K))
     q_rows = rejected * V * esize if wl.q is not None else 0
     gathers = B * K * 2 * 32
@@ -402,17 +424,17 @@ def run_ours(args):
     import paper_2607_25852_gb300 as spec
 
     wl = make_inputs(args, rank, device)
-    R = wl.rows
     step = Step(wl, device)
+    R = step.rows  # verified positions per step: the chosen budget T*
     stream = torch.cuda.current_stream()
 
     for _ in range(max(args.warmup, 3)):
         step.run()
     torch.cuda.synchronize()
     assert int(step.status.item()) == 0, "device reported an input error"
-    assert int(step.chosen.item()) == R, "the flat cost table should select the full block"
+    assert int(step.chosen.item()) == R, "the allocation changed between steps"
     acc = step.acc.cpu().numpy()
-    alg = algorithmic_bytes(wl, acc)
+    alg = algorithmic_bytes(wl, acc, R)
 
     # ---- device-timed region ----
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -510,9 +532,10 @@ def run_ours(args):
     # measured too.
     e2e = None
     if not args.no_e2e:
-        host = {k: getattr(wl, k).cpu().pin_memory() for k in
-                ("conf", "logits", "drafts", "q", "seeds", "request_ids", "pos_base", "last_tokens",
-                 "hidden") if getattr(wl, k) is not None}
+        src = dict(conf=wl.conf, logits=step.logits, drafts=wl.drafts, q=wl.q, seeds=wl.seeds,
+                   request_ids=wl.request_ids, pos_base=wl.pos_base, last_tokens=wl.last_tokens,
+                   hidden=step.hidden)  # the packed rows of the step's allocation
+        host = {k: v.cpu().pin_memory() for k, v in src.items() if v is not None}
         dev_in = {k: torch.empty_like(v, device=device) for k, v in host.items()}
         dev_in.setdefault("q", None)
         outs_host = [torch.empty_like(t, device="cpu").pin_memory() for t in (step.acc, step.tok, step.ctok, step.coff)]
@@ -551,7 +574,7 @@ def run_ours(args):
             # what crosses the link in place: every logits row, the q row at
             # each rejection and the q(z) sectors, the committed hidden rows,
             # and the small inputs that are copied
-            ab = algorithmic_bytes(wl, step.acc.cpu().numpy())
+            ab = algorithmic_bytes(wl, step.acc.cpu().numpy(), R)
             small_bytes = sum(t.numel() * t.element_size() for k, t in host.items() if k not in big)
             h2d_moved = (ab["logits"] + ab["q_rows"] + (wl.B * wl.K * 32 if wl.q is not None else 0)
                          + ab["commit"] // 2 + small_bytes)
@@ -600,7 +623,9 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
         "config": {"workload": f"{wl.name}: B={wl.B} K={wl.K} V={wl.V} {wl.dtype} logits, "
                                f"t={wl.temperature}, q {'bf16 [B,K,V]' if wl.q is not None else 'one-hot'}, "
-                               f"H={wl.H}; D-cut ratios 1/4..1 with a flat cost table (T*={R})",
+                               f"H={wl.H}; " + (f"D-cut over T = 64..1024 with cost 1 + 0.004 max(0, T - 256) "
+                                                 f"(T*={R})" if wl.name == "alloc" else
+                                                 f"D-cut ratios 1/4..1 with a flat cost table (T*={R})"),
                    "rows_per_step": R,
                    "l2": (f"inputs larger than L2 ({alg['logits'] / 1e6:.1f} MB logits per step, no flush)"
                           if flush is None else
