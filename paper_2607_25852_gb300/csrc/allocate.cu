@@ -24,6 +24,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "spec_internal.cuh"
 
@@ -117,6 +118,10 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_kernel(const AllocLaun
   // The next kernel (the streaming pass) may launch now: it waits for this
   // one's completion before it reads the depths and row offsets.
   pdl_launch_dependents();
+  // This kernel starts while the previous one on the stream drains; it reads
+  // its inputs, and overwrites the arrays the previous round's kernels read,
+  // only once that kernel has completed.
+  pdl_wait_prerequisites();
 
   // ---- every global input in one round trip, coalesced ----
   for (int q = tid; q < BK; q += kAllocThreads) {
@@ -316,6 +321,10 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
   // The next kernel (the streaming pass) may launch now: it waits for this
   // one's completion before it reads the depths and row offsets.
   pdl_launch_dependents();
+  // This kernel starts while the previous one on the stream drains; it reads
+  // its inputs, and overwrites the arrays the previous round's kernels read,
+  // only once that kernel has completed.
+  pdl_wait_prerequisites();
 
   // ---- every global input in one round trip ----
   if (tid < NK) {
@@ -482,16 +491,30 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
 bool allocate_is_small(int B, int K) { return B <= kSmallSlots && (long long)B * K <= kSmallSlots; }
 
 cudaError_t launch_allocate(const AllocLaunch& p, cudaStream_t stream) {
+  cudaError_t err;
   if (allocate_is_small(p.B, p.K)) {
-    allocate_small_kernel<<<1, kAllocThreads, 0, stream>>>(p);
-    return cudaGetLastError();
+    err = launch_after_previous(allocate_small_kernel, dim3(1), dim3(kAllocThreads), 0, stream, p);
+    return err != cudaSuccess ? err : cudaGetLastError();
   }
+  // The dynamic shared memory limit is raised once per device, to the
+  // largest size asked for so far.
   const size_t smem = allocate_smem_bytes(p.B, p.K);
-  cudaError_t err = cudaFuncSetAttribute(allocate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+  constexpr int kMaxDevices = 64;
+  static std::atomic<size_t> raised[kMaxDevices];
+  int dev = -1;
+  err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  allocate_kernel<<<1, kAllocThreads, smem, stream>>>(p);
-  return cudaGetLastError();
+  if (dev < 0 || dev >= kMaxDevices || raised[dev].load(std::memory_order_relaxed) < smem) {
+    err = cudaFuncSetAttribute(allocate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (err != cudaSuccess) return err;
+    if (dev >= 0 && dev < kMaxDevices) {
+      size_t cur = raised[dev].load(std::memory_order_relaxed);
+      while (cur < smem && !raised[dev].compare_exchange_weak(cur, smem)) {
+      }
+    }
+  }
+  err = launch_after_previous(allocate_kernel, dim3(1), dim3(kAllocThreads), smem, stream, p);
+  return err != cudaSuccess ? err : cudaGetLastError();
 }
 
 }  // namespace spec
