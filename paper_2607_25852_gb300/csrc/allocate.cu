@@ -10,8 +10,9 @@
 // then lower request index.  Keys are unique.
 //
 // Batches of at most 1024 requests and 1024 draft positions take
-// allocate_small_kernel (below): a bitonic sort of the draft keys alone.
-// Larger batches take allocate_kernel:
+// allocate_small_kernel (below), which sorts the draft keys alone: a merge
+// tree over the per-request runs padded to a power of two when they fit in
+// 1024 slots, else a bitonic sort.  Larger batches take allocate_kernel:
 // because s_{i,k} is non-increasing in k, each request's K+1 keys already form
 // a run sorted in descending order.  A merge tree of ceil(log2 B) levels sorts
 // the B runs: at every level each key finds its place in the merged pair by
@@ -339,11 +340,11 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
   __syncthreads();
 
   // ---- Eq. (dcut-score): fp32 prefix products, request i in thread i ----
-  // Each request's keys go to a run of KP = next power of two >= K slots,
-  // padded with key 0 (below every real key), in descending order for even i
-  // and ascending order for odd i when B * KP <= 1024: the runs are then the
-  // sorted, alternating blocks that the bitonic network's first log2(KP)
-  // levels would produce, and those levels are skipped.
+  // When B * KP <= 1024 (KP = the next power of two >= K), request i's keys
+  // fill run i of KP slots in descending order (s is non-increasing in k),
+  // and the slots past K, and the runs past B, hold pad keys: unique, below
+  // every real key, descending within a run.  A merge tree then sorts the
+  // 1024 slots.  Otherwise the keys are staged unsorted for a bitonic sort.
   const int KP = K <= 1 ? 1 : 1 << (32 - __clz(K - 1));
   const bool runs = B * KP <= kSmallSlots;
   // Keys are staged with a row of RL slots per request at the odd stride
@@ -369,38 +370,63 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
         }
         c = __fadd_rn(c, 0.0f);  // -0 counts as +0 (its sign bit would break the key order)
         s = __fmul_rn(s, c);
-        const int slot = tid * RS + (runs && (tid & 1) ? KP - k : k - 1);
-        stage[slot] = position_key(s, k, tid);
+        stage[tid * RS + k - 1] = position_key(s, k, tid);
       }
     }
-    if (runs)
-      for (int k = K + 1; k <= KP; ++k) stage[tid * RS + ((tid & 1) ? KP - k : k - 1)] = 0ull;
   }
   __syncthreads();
 
-  // ---- bitonic sort of the draft keys, descending ----
-  const int NS = runs ? B * KP : NK;  // occupied slots
-  unsigned long long x = tid < NS ? stage[(tid / RL) * RS + tid % RL] : 0ull;
-  __syncthreads();  // the staging area is the exchange buffer from here on
-  int buf = 1;
+  unsigned long long x;
+  if (runs) {
+    // slot u = i * KP + (k - 1); a pad key is 1024 - u (real keys are above
+    // 0xFBFF0000 even at s = 0)
+    x = (tid / KP < B && tid % KP < K) ? stage[(tid / KP) * RS + tid % KP] : (unsigned long long)(kSmallSlots - tid);
+    __syncthreads();  // the staging area holds the merge buffers from here on
+    // ---- merge tree, descending: at the level of runs of L keys, a key's
+    // place in the merged pair is its index in its run plus the number of
+    // keys of the partner run above it (keys are unique), found by a
+    // branch-free binary search of log2(L) + 1 shared-memory probes ----
+    auto word = [](int e) { return 8u * (uint32_t)e; };
+    uint32_t src = (uint32_t)__cvta_generic_to_shared(&sh_x[0][0]);
+    uint32_t dst = (uint32_t)__cvta_generic_to_shared(&sh_x[1][0]);
+    sts_u64(src + word(tid), x);
+    __syncthreads();
+    for (int L = KP; L < kSmallSlots; L <<= 1) {
+      const int partner = (tid ^ L) & ~(L - 1);
+      int c = 0;
+      for (int step = L >> 1; step > 0; step >>= 1)
+        if (lds_u64(src + word(partner + c + step - 1)) > x) c += step;
+      if (lds_u64(src + word(partner + c)) > x) ++c;
+      sts_u64(dst + word((tid & ~(2 * L - 1)) + (tid & (L - 1)) + c), x);
+      __syncthreads();
+      const uint32_t t = src;
+      src = dst;
+      dst = t;
+      x = lds_u64(src + word(tid));
+    }
+  } else {
+    // ---- bitonic sort of the draft keys, descending ----
+    x = tid < NK ? stage[(tid / RL) * RS + tid % RL] : 0ull;
+    __syncthreads();  // the staging area is the exchange buffer from here on
+    int buf = 1;
 #pragma unroll
-  for (int k = 2; k <= kSmallSlots; k <<= 1) {
-    if (runs && k <= KP) continue;  // the runs are sorted blocks of KP already
+    for (int k = 2; k <= kSmallSlots; k <<= 1) {
 #pragma unroll
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      unsigned long long y;
-      if (j >= 32) {
-        sh_x[buf][tid] = x;
-        __syncthreads();
-        y = sh_x[buf][tid ^ j];
-        buf ^= 1;
-      } else {
-        y = shfl_xor_u64(x, j);
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        unsigned long long y;
+        if (j >= 32) {
+          sh_x[buf][tid] = x;
+          __syncthreads();
+          y = sh_x[buf][tid ^ j];
+          buf ^= 1;
+        } else {
+          y = shfl_xor_u64(x, j);
+        }
+        // blocks of k alternate direction (descending first); the lower
+        // index of a pair keeps the larger key in a descending block
+        const bool take_max = ((tid & k) == 0) == ((tid & j) == 0);
+        x = take_max ? (x > y ? x : y) : (x < y ? x : y);
       }
-      // blocks of k alternate direction (descending first); the lower index
-      // of a pair keeps the larger key in a descending block
-      const bool take_max = ((tid & k) == 0) == ((tid & j) == 0);
-      x = take_max ? (x > y ? x : y) : (x < y ? x : y);
     }
   }
   // x: the draft key of rank tid (tid < NK)
