@@ -280,7 +280,7 @@ __global__ void __launch_bounds__(32) shard_decide_kernel(const ShardLaunch p) {
   __shared__ float sh_pz[kMaxRows];
   __shared__ float sh_lq[kMaxRows];
   const ReqShape rs = request_shape(p, i);
-  const DecidePre pre = decide_prefetch(p, i);
+  const DecidePre pre = decide_prefetch<ShardLaunch, false, !kGreedy>(p, i);
   const int n = rs.n;
   const long long row0 = rs.row0;
 #pragma unroll

@@ -76,17 +76,21 @@ VerifyGeometry verify_geometry(int B, int K, int V) {
 // the target logit and the draft probability at each draft, and runs the
 // decision chain.  Only one warp of a CTA decides at a time (its shared arrays
 // are per CTA).
+// The decision arrays of a CTA (row statistics, drafts, p_j(z)), kept after
+// the decision for the outputs written later.
+__shared__ float sh_m[kMaxRows];
+__shared__ float sh_S[kMaxRows];
+__shared__ int32_t sh_g[kMaxRows];
+__shared__ int32_t sh_z[kMaxRows];
+__shared__ float sh_pz[kMaxRows];
+__device__ __forceinline__ DecideArrays decide_arrays() { return DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}; }
+
 template <typename T, bool kGreedy>
 __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre,
                                             bool outputs, ReqRec* rec_dst) {
   const int K = p.K, V = p.V, NC = p.NC;
   const float c2 = p.c2;
   const int lane = threadIdx.x & 31;
-  __shared__ float sh_m[kMaxRows];
-  __shared__ float sh_S[kMaxRows];
-  __shared__ int32_t sh_g[kMaxRows];
-  __shared__ int32_t sh_z[kMaxRows];
-  __shared__ float sh_pz[kMaxRows];
   const int n = rs.n;
   const long long row0 = rs.row0;
 
@@ -158,7 +162,7 @@ __device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqSha
     if (sh_z[j] < 0 || sh_z[j] >= V) bad = 1;
   bad = __any_sync(0xFFFFFFFFu, bad);
   __syncwarp();
-  decide_chain<kGreedy>(p, i, rs, pre, DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}, lz, qz, bad, outputs, rec_dst);
+  decide_chain<kGreedy>(p, i, rs, pre, decide_arrays(), lz, qz, bad, outputs, rec_dst);
   if (kGreedy && lane == 0) p.req_count[i] = 0u;  // leave the workspace zeroed for the next call
   __syncwarp();
 }
@@ -248,14 +252,25 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   const int V = p.V;
   const int warp = threadIdx.x >> 5;
   __shared__ ReqRec sh_rec;
+  // The request's shape, its drafts and seeds and the acceptance variates do
+  // not depend on the streaming kernel: they are loaded (through L2) and drawn
+  // while it drains.  Their producers completed before this grid could
+  // launch: the allocator (the streaming CTAs waited for it before they let
+  // this grid start) and the caller's earlier work.
+  const ReqShape rs = request_shape<VerifyLaunch, true>(p, i);
+  DecidePre pre{};
+  if (warp == 0) pre = decide_prefetch<VerifyLaunch, true, true>(p, i);
   pdl_wait_prerequisites();  // the row partials of the streaming kernel
   pdl_launch_dependents();   // the commit kernel waits for this grid in turn
-  // The request's decision chain (every CTA of the request runs it, chunk 0
-  // writes the outputs): which row to sample, and how.
-  if (warp == 0) decide_request<T, false>(p, i, request_shape(p, i), decide_prefetch(p, i), cs == 0, &sh_rec);
+  // The request's decision chain (every CTA of the request runs it; the last
+  // CTA to finish the race writes the outputs): which row to sample, and how.
+  if (warp == 0) decide_request<T, false>(p, i, rs, pre, false, &sh_rec);
   __syncthreads();
   const ReqRec rec = sh_rec;
-  if (rec.flags & 1) return;  // bad input: the decision wrote the outputs
+  if (rec.flags & 1) {  // bad input: chunk 0 writes the flagged outputs
+    if (cs == 0 && warp == 0) write_decision<false>(p, i, rs, decide_arrays(), 0, 1);
+    return;
+  }
   // A record that could not come from a consistent decision is refused
   // rather than used to read outside the inputs.
   if (rec.a < 0 || rec.a > p.K || rec.srow < 0 || rec.srow >= p.R_max || rec.z_excl < -1 || rec.z_excl >= V ||
@@ -312,6 +327,7 @@ __global__ void __launch_bounds__(kSampleThreads, 4) sample_kernel(const VerifyL
   if (!sh_last) return;
 
   __threadfence();
+  if (warp == 1) write_decision<false>(p, i, rs, decide_arrays(), rec.a, 0);  // the token at a comes last
   if (warp == 0) {
     // the partials of all chunks at once, one lane each
     const int lane = threadIdx.x & 31;

@@ -619,15 +619,22 @@ struct ReqShape {
   bool valid;
 };
 
-template <class L>
+// kL2: load through L2 only (loads a kernel issues before its grid-dependency
+// wait, of data that kernels before the previous one wrote).
+template <bool kL2, typename E>
+__device__ __forceinline__ E load_in(const E* a) {
+  return kL2 ? __ldcg(a) : __ldg(a);
+}
+
+template <class L, bool kL2 = false>
 __device__ __forceinline__ ReqShape request_shape(const L& p, int i) {
-  const int n_in = p.depth ? __ldg(p.depth + i) : p.K;
+  const int n_in = p.depth ? load_in<kL2>(p.depth + i) : p.K;
   long long off0 = (long long)i * (p.K + 1), off1 = off0 + n_in + 1;
   if (p.row_offsets) {
-    off0 = __ldg(p.row_offsets + i);
-    off1 = __ldg(p.row_offsets + i + 1);
+    off0 = load_in<kL2>(p.row_offsets + i);
+    off1 = load_in<kL2>(p.row_offsets + i + 1);
   }
-  const long long pos = __ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
+  const long long pos = load_in<kL2>(reinterpret_cast<const long long*>(p.pos_base) + i);
   ReqShape s;
   s.valid = n_in >= 0 && n_in <= p.K && off0 >= 0 && off1 == off0 + n_in + 1 && off1 <= p.R_max &&
             pos >= 0 && pos + n_in <= 0xFFFFFFFFLL;
@@ -636,25 +643,35 @@ __device__ __forceinline__ ReqShape request_shape(const L& p, int i) {
   return s;
 }
 
-// What a decision reads first (seeds and draft tokens), loaded by the
-// deciding warp before it learns whether it decides, so that these loads
-// overlap the arrival atomic.  z[u] is draft j = lane + 32u.
+// What a decision needs that the rows' statistics do not decide: seeds,
+// draft tokens and (kDraws) the acceptance variates, prepared by the deciding
+// warp before the statistics are complete (before the arrival atomic, or
+// before the grid-dependency wait).  z[u] and u[u] belong to draft
+// j = lane + 32u.
 struct DecidePre {
   uint32_t pos;
   unsigned long long seed, req;
   int32_t z[(kMaxRows + 31) / 32];
+  float u[(kMaxRows + 31) / 32];
 };
-template <class L>
+template <class L, bool kL2 = false, bool kDraws = false>
 __device__ __forceinline__ DecidePre decide_prefetch(const L& p, int i) {
   const int lane = threadIdx.x & 31;
   DecidePre pre;
-  pre.pos = (uint32_t)__ldg(reinterpret_cast<const long long*>(p.pos_base) + i);
-  pre.seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
-  pre.req = __ldg(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
+  pre.pos = (uint32_t)load_in<kL2>(reinterpret_cast<const long long*>(p.pos_base) + i);
+  pre.seed = load_in<kL2>(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
+  pre.req = load_in<kL2>(reinterpret_cast<const unsigned long long*>(p.request_ids) + i);
 #pragma unroll
   for (int u = 0; u < (kMaxRows + 31) / 32; ++u) {
     const int j = lane + 32 * u;
-    pre.z[u] = j < p.K ? __ldg(p.drafts + (size_t)i * p.K + j) : 0;
+    pre.z[u] = j < p.K ? load_in<kL2>(p.drafts + (size_t)i * p.K + j) : 0;
+    pre.u[u] = 1.0f;
+    if (kDraws && j < p.K) {
+      // u_j, the uniform of draft j's acceptance test: 24 bits, exactly
+      const uint4 w = philox(draw_counter(pre.pos + (uint32_t)j, pre.req, SPEC_PURPOSE_ACCEPT, 0u),
+                             (uint32_t)pre.seed, (uint32_t)(pre.seed >> 32));
+      pre.u[u] = (float)(w.x >> 8) * 0x1p-24f;
+    }
   }
   return pre;
 }
@@ -680,6 +697,49 @@ struct DecideArrays {
 // `outputs`: write the request's outputs (several CTAs may run the same
 // decision; one of them writes); `rec_dst` (t > 0): where the record of the
 // row to sample goes.
+// The decision's outputs, one warp, from the decision arrays (sh.z the
+// drafts, sh.pz p_j(z), sh.m / sh.S or sh.m the row statistics): the
+// committed prefix (the sampled or argmax token at position a is written
+// apart), -1 past it, a, p(z) and the row statistics; for a flagged request
+// -1 tokens, a = 0 and zero probabilities.
+template <bool kGreedy, class L>
+__device__ __forceinline__ void write_decision(const L& p, int i, const ReqShape& rs, const DecideArrays& sh, int a,
+                                               int bad) {
+  const int K = p.K, n = rs.n;
+  const int lane = threadIdx.x & 31;
+  int32_t* tok = p.out_tokens + (size_t)i * (K + 1);
+  if (bad) {
+    if (lane == 0) report(p.status, SPEC_ERR_BAD_INPUT);
+    for (int j = lane; j <= K; j += 32) tok[j] = -1;
+    if (lane == 0) p.accepted_len[i] = 0;
+    if (p.p_draft)
+      for (int j = lane; j < K; j += 32) p.p_draft[(size_t)i * K + j] = 0.0f;
+    return;
+  }
+  for (int j = lane; j <= K; j += 32) {
+    if (j < a) tok[j] = sh.z[j];
+    else if (j > a) tok[j] = -1;
+  }
+  if (lane == 0) p.accepted_len[i] = a;
+  if (p.p_draft)
+    for (int j = lane; j < K; j += 32) p.p_draft[(size_t)i * K + j] = j < n ? sh.pz[j] : 0.0f;
+  if (p.row_stats) {
+    for (int j = lane; j <= n; j += 32) {
+      float2 st;
+      if (kGreedy) {
+        st = make_float2(sh.m[j], 0.0f);
+      } else {
+        // ln S relative to the exact max / t: S is kept relative to
+        // fl(m * c2), and fmaf gives m * c2 - fl(m * c2) exactly
+        const float c2 = p.c2;
+        const float resid = fmaf(sh.m[j], c2, -(sh.m[j] * c2));
+        st = make_float2(sh.m[j] * p.inv_t, (log2f(sh.S[j]) - resid) * 0.69314718055994531f);
+      }
+      reinterpret_cast<float2*>(p.row_stats)[rs.row0 + j] = st;
+    }
+  }
+}
+
 template <bool kGreedy, class L>
 __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& rs, const DecidePre& pre,
                                              const DecideArrays& sh, const float (&lz)[(kMaxRows + 31) / 32],
@@ -691,7 +751,6 @@ __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& 
   const int n = rs.n;
   const long long row0 = rs.row0;
   const uint32_t pos = pre.pos;
-  const unsigned long long seed = pre.seed, req = pre.req;
   float* sh_m = sh.m;
   float* sh_S = sh.S;
   int32_t* sh_g = sh.g;
@@ -718,10 +777,7 @@ __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& 
           r = fminf(1.0f, pz / qz[u]);
         else
           r = pz > 0.0f ? 1.0f : 0.0f;
-        const uint4 w = philox(draw_counter(pos + (uint32_t)j, req, SPEC_PURPOSE_ACCEPT, 0u), (uint32_t)seed,
-                               (uint32_t)(seed >> 32));
-        const float uu = (float)(w.x >> 8) * 0x1p-24f;  // exact
-        reject = !(uu < r);
+        reject = !(pre.u[u] < r);  // u_j drawn by decide_prefetch
         sh_pz[j] = pz;
       }
       if (reject) first_reject = min(first_reject, j);
@@ -733,37 +789,7 @@ __device__ __forceinline__ void decide_chain(const L& p, int i, const ReqShape& 
 
   const int a = bad ? 0 : first_reject;
   int32_t* tok = p.out_tokens + (size_t)i * (K + 1);
-  if (!outputs) {
-    // another CTA writes this request's outputs
-  } else if (bad) {
-    if (lane == 0) report(p.status, SPEC_ERR_BAD_INPUT);
-    for (int j = lane; j <= K; j += 32) tok[j] = -1;
-    if (lane == 0) p.accepted_len[i] = 0;
-    if (p.p_draft)
-      for (int j = lane; j < K; j += 32) p.p_draft[(size_t)i * K + j] = 0.0f;
-  } else {
-    for (int j = lane; j <= K; j += 32) {
-      if (j < a) tok[j] = sh_z[j];
-      else if (j > a) tok[j] = -1;
-    }
-    if (lane == 0) p.accepted_len[i] = a;
-    if (p.p_draft)
-      for (int j = lane; j < K; j += 32) p.p_draft[(size_t)i * K + j] = j < n ? sh_pz[j] : 0.0f;
-    if (p.row_stats) {
-      for (int j = lane; j <= n; j += 32) {
-        float2 st;
-        if (kGreedy) {
-          st = make_float2(sh_m[j], 0.0f);
-        } else {
-          // ln S relative to the exact max / t: S is kept relative to
-          // fl(m * c2), and fmaf gives m * c2 - fl(m * c2) exactly
-          const float resid = fmaf(sh_m[j], c2, -(sh_m[j] * c2));
-          st = make_float2(sh_m[j] * p.inv_t, (log2f(sh_S[j]) - resid) * 0.69314718055994531f);
-        }
-        reinterpret_cast<float2*>(p.row_stats)[row0 + j] = st;
-      }
-    }
-  }
+  if (outputs) write_decision<kGreedy>(p, i, rs, sh, a, bad);
   if (lane == 0) {
     if (kGreedy) {
       if (!bad && outputs) tok[a] = sh_g[a];
