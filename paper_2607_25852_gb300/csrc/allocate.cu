@@ -307,6 +307,26 @@ __device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long x,
   return ((unsigned long long)hi << 32) | lo;
 }
 
+// One level of the small kernel's merge tree over kSmallSlots keys in shared
+// memory (src), runs of L keys merged in pairs into dst; x is the calling
+// thread's key at slot tid, and on return the key at slot tid of the merged
+// order (src and dst swapped).
+template <int L>
+__device__ __forceinline__ void merge_level(unsigned long long& x, int tid, uint32_t& src, uint32_t& dst) {
+  const uint32_t partner = src + 8u * (uint32_t)((tid ^ L) & ~(L - 1));
+  int c = 0;
+#pragma unroll
+  for (int step = L >> 1; step > 0; step >>= 1)
+    if (lds_u64(partner + 8u * (uint32_t)(c + step - 1)) > x) c += step;
+  if (lds_u64(partner + 8u * (uint32_t)c) > x) ++c;
+  sts_u64(dst + 8u * (uint32_t)((tid & ~(2 * L - 1)) + (tid & (L - 1)) + c), x);
+  __syncthreads();
+  const uint32_t t = src;
+  src = dst;
+  dst = t;
+  x = lds_u64(src + 8u * (uint32_t)tid);
+}
+
 __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const AllocLaunch p) {
   __shared__ float sh_conf[2 * kSmallSlots];               // [i][k] at i * (K | 1) + k
   __shared__ int32_t sh_drafts[kSmallSlots];
@@ -386,23 +406,23 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
     // place in the merged pair is its index in its run plus the number of
     // keys of the partner run above it (keys are unique), found by a
     // branch-free binary search of log2(L) + 1 shared-memory probes ----
-    auto word = [](int e) { return 8u * (uint32_t)e; };
     uint32_t src = (uint32_t)__cvta_generic_to_shared(&sh_x[0][0]);
     uint32_t dst = (uint32_t)__cvta_generic_to_shared(&sh_x[1][0]);
-    sts_u64(src + word(tid), x);
+    sts_u64(src + 8u * (uint32_t)tid, x);
     __syncthreads();
-    for (int L = KP; L < kSmallSlots; L <<= 1) {
-      const int partner = (tid ^ L) & ~(L - 1);
-      int c = 0;
-      for (int step = L >> 1; step > 0; step >>= 1)
-        if (lds_u64(src + word(partner + c + step - 1)) > x) c += step;
-      if (lds_u64(src + word(partner + c)) > x) ++c;
-      sts_u64(dst + word((tid & ~(2 * L - 1)) + (tid & (L - 1)) + c), x);
-      __syncthreads();
-      const uint32_t t = src;
-      src = dst;
-      dst = t;
-      x = lds_u64(src + word(tid));
+    // the levels from runs of KP on, each unrolled for its L
+    switch (31 - __clz(KP)) {
+      case 0: merge_level<1>(x, tid, src, dst); [[fallthrough]];
+      case 1: merge_level<2>(x, tid, src, dst); [[fallthrough]];
+      case 2: merge_level<4>(x, tid, src, dst); [[fallthrough]];
+      case 3: merge_level<8>(x, tid, src, dst); [[fallthrough]];
+      case 4: merge_level<16>(x, tid, src, dst); [[fallthrough]];
+      case 5: merge_level<32>(x, tid, src, dst); [[fallthrough]];
+      case 6: merge_level<64>(x, tid, src, dst); [[fallthrough]];
+      case 7: merge_level<128>(x, tid, src, dst); [[fallthrough]];
+      case 8: merge_level<256>(x, tid, src, dst); [[fallthrough]];
+      case 9: merge_level<512>(x, tid, src, dst); [[fallthrough]];
+      default: break;
     }
   } else {
     // ---- bitonic sort of the draft keys, descending ----
@@ -483,17 +503,31 @@ __global__ void __launch_bounds__(kAllocThreads) allocate_small_kernel(const All
   }
   __syncthreads();
 
-  // ---- row offsets: exclusive scan of (n_i + 1) ----
-  const int cnt = tid < B ? depth[tid] + 1 : 0;
-  const long long rincl = block_inclusive_scan((long long)cnt, warp_tot);
-  if (tid < B) {
-    offsets[tid] = (int)(rincl - cnt);
-    p.row_offsets_out[tid] = (int)(rincl - cnt);
-    p.depth_out[tid] = cnt - 1;
-  }
-  if (tid == 0) {
-    p.row_offsets_out[B] = T;  // sum of (n_i + 1): the T kept positions
-    *p.chosen_T_out = T;
+  // ---- row offsets: exclusive scan of (n_i + 1), one warp: lane l takes
+  // the requests [l * m, (l + 1) * m) in order, m = ceil(B / 32) ----
+  if (tid < 32) {
+    const int m = (B + 31) >> 5;
+    const int i0 = min(B, tid * m), i1 = min(B, i0 + m);
+    int sum = 0;
+    for (int i = i0; i < i1; ++i) sum += depth[i] + 1;
+    int incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (tid >= o) incl += y;
+    }
+    int off = incl - sum;
+    for (int i = i0; i < i1; ++i) {
+      const int n = depth[i];
+      offsets[i] = off;
+      p.row_offsets_out[i] = off;
+      p.depth_out[i] = n;
+      off += n + 1;
+    }
+    if (tid == 0) {
+      p.row_offsets_out[B] = T;  // sum of (n_i + 1): the T kept positions
+      *p.chosen_T_out = T;
+    }
   }
   __syncthreads();
 
