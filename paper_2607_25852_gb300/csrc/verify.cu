@@ -86,7 +86,7 @@ __shared__ float sh_pz[kMaxRows];
 __device__ __forceinline__ DecideArrays decide_arrays() { return DecideArrays{sh_m, sh_S, sh_g, sh_z, sh_pz}; }
 
 template <typename T, bool kGreedy>
-__device__ __noinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre,
+__device__ __forceinline__ void decide_request(const VerifyLaunch& p, int i, ReqShape rs, const DecidePre& pre,
                                             bool outputs, ReqRec* rec_dst) {
   const int K = p.K, V = p.V, NC = p.NC;
   const float c2 = p.c2;
