@@ -123,9 +123,8 @@ __device__ __forceinline__ uint64_t global_ns() {
   return t;
 }
 // Wait for the phase with parity `parity`; false (and SPEC_ERR_TIMEOUT) after
-// about a second.
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* status) {
-  if (mbar_try_wait(bar, parity)) return true;
+// about a second.  The bounded loop is out of line; the first try is not.
+__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, int32_t* status) {
   const uint64_t t0 = global_ns();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -134,6 +133,9 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* 
       return false;
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int32_t* status) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, status);
 }
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
