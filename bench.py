@@ -662,6 +662,7 @@ def run_ours(args):
         "step_ms_p10_p50_p90": [float(np.percentile(step_ms, p)) for p in (10, 50, 90)],
         "step_ms_how": "single steps, each bracketed by events (no overlap with the step before)",
         "mean_accepted": float(acc.mean()),
+        "accepted_histogram": [int(x) for x in np.bincount(acc, minlength=wl.K + 1)],
         "clocks": clocks.summary(),
         "e2e": e2e,
         "graph": graph,

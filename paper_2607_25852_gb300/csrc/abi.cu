@@ -4,17 +4,13 @@
 // Nothing here allocates device memory, synchronises a stream or reads device
 // memory, so every entry point is stream-ordered.
 #include <math.h>
-#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
 
 #include "spec_internal.cuh"
 
 namespace {
 
-struct NvtxRange {
-  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
-  ~NvtxRange() { nvtxRangePop(); }
-};
+using spec::NvtxRange;
 
 cudaEvent_t g_profile_before = nullptr;
 cudaEvent_t g_profile_after = nullptr;

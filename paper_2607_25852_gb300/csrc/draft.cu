@@ -539,6 +539,7 @@ extern "C" int spec_draft(const void* logits, int logits_dtype, int B, int K, in
                           const uint64_t* seeds, const uint64_t* request_ids, const int64_t* pos_base,
                           int32_t* drafts_out, float* conf_out, float* scores_out, float* row_stats_out,
                           int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  spec::NvtxRange range("spec_draft");
   if (B < 1 || K < 1 || K > SPEC_MAX_DRAFTS || V < 1 || V >= SPEC_MAX_VOCAB || (long long)B * K > (1LL << 28))
     return SPEC_ERR_INVALID_ARG;
   if ((logits_dtype != SPEC_BF16 && logits_dtype != SPEC_F32) || !(tau >= 0.0f) || isinf(tau))

@@ -851,6 +851,7 @@ extern "C" int spec_markov_draft(const void* U, int u_dtype, const void* W1, con
                                  const uint64_t* request_ids, const int64_t* pos_base, int32_t* drafts_out,
                                  float* conf_out, float* scores_out, float* row_stats_out, int32_t* status,
                                  void* ws, size_t ws_bytes, cudaStream_t stream) {
+  spec::NvtxRange range("spec_markov_draft");
   using namespace spec;
   if (!markov_shape_ok(B, K, V, r) || u_dtype != SPEC_BF16 || !(tau >= 0.0f) || isinf(tau))
     return SPEC_ERR_INVALID_ARG;

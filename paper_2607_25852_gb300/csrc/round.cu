@@ -125,6 +125,7 @@ extern "C" int spec_graph_destroy(void* exec) {
 
 extern "C" int spec_select_round(const int32_t* chosen_T, int M, const int32_t* cand_T, void* const* graphs,
                                  int32_t* launched_out, int32_t* status, cudaStream_t stream) {
+  spec::NvtxRange range("spec_select_round");
   if (!chosen_T || M < 1 || M > SPEC_MAX_CANDIDATES || !cand_T || !graphs) return SPEC_ERR_INVALID_ARG;
   spec::SelectParams p{};
   p.M = M;
@@ -142,6 +143,7 @@ extern "C" int spec_select_round(const int32_t* chosen_T, int M, const int32_t* 
 
 extern "C" int spec_pack_rows(const void* src, size_t row_bytes, int B, int K, const int32_t* row_offsets,
                               void* dst, int R_dst, int32_t* status, cudaStream_t stream) {
+  spec::NvtxRange range("spec_pack_rows");
   if (!src || !dst || !row_offsets || row_bytes == 0 || B < 1 || K < 0 || K > SPEC_MAX_DRAFTS || R_dst < 1 ||
       (long long)B * (K + 1) > (1LL << 28))
     return SPEC_ERR_INVALID_ARG;

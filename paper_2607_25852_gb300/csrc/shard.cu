@@ -744,6 +744,7 @@ extern "C" int spec_shard_stats(const void* logits_shard, int logits_dtype, cons
                                 int B, int K, int V, int v_begin, int V_shard, float temperature,
                                 const int64_t* pos_base, void* stats_out, int32_t* status, void* ws,
                                 size_t ws_bytes, cudaStream_t stream) {
+  spec::NvtxRange range("spec_shard_stats");
   if (!spec::shard_shape_ok(B, K, V, v_begin, V_shard)) return SPEC_ERR_INVALID_ARG;
   if ((logits_dtype != SPEC_BF16 && logits_dtype != SPEC_F32) || !(temperature >= 0.0f) || isinf(temperature))
     return SPEC_ERR_INVALID_ARG;
@@ -793,6 +794,7 @@ extern "C" int spec_shard_decide(const void* stats, int S, const int32_t* row_of
                                  const uint64_t* seeds, const uint64_t* request_ids, const int64_t* pos_base,
                                  int32_t* accepted_len_out, int32_t* out_tokens, float* p_draft_out,
                                  float* row_stats_out, void* decisions_out, int32_t* status, cudaStream_t stream) {
+  spec::NvtxRange range("spec_shard_decide");
   if (!spec::shard_shape_ok(B, K, V, 0, V) || S < 1 || S > V) return SPEC_ERR_INVALID_ARG;
   if (!(temperature >= 0.0f) || isinf(temperature)) return SPEC_ERR_INVALID_ARG;
   if (!stats || (K > 0 && !draft_tokens) || !seeds || !request_ids || !pos_base || !accepted_len_out ||
@@ -830,6 +832,7 @@ extern "C" int spec_shard_sample(const void* logits_shard, int logits_dtype, con
                                  const void* decisions, int B, int K, int V, int v_begin, int V_shard,
                                  float temperature, const uint64_t* seeds, const uint64_t* request_ids,
                                  void* race_out, int32_t* status, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  spec::NvtxRange range("spec_shard_sample");
   if (!spec::shard_shape_ok(B, K, V, v_begin, V_shard)) return SPEC_ERR_INVALID_ARG;
   if ((logits_dtype != SPEC_BF16 && logits_dtype != SPEC_F32) || !(temperature >= 0.0f) || isinf(temperature))
     return SPEC_ERR_INVALID_ARG;
@@ -884,6 +887,7 @@ extern "C" int spec_shard_finish(const void* races, int S, const void* decisions
                                  float temperature, const uint64_t* seeds, const uint64_t* request_ids,
                                  int32_t* accepted_len_out, int32_t* out_tokens, int32_t* status,
                                  cudaStream_t stream) {
+  spec::NvtxRange range("spec_shard_finish");
   if (!spec::shard_shape_ok(B, K, V, 0, V) || S < 1 || S > V) return SPEC_ERR_INVALID_ARG;
   if (!(temperature >= 0.0f) || isinf(temperature)) return SPEC_ERR_INVALID_ARG;
   if (temperature == 0.0f) return SPEC_OK;

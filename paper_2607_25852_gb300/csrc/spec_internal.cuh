@@ -4,6 +4,7 @@
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
 
 #include "spec.h"
@@ -80,6 +81,13 @@ __device__ __forceinline__ float load_any(const void* base, int dtype, int64_t i
 // launching / wait until the previous kernel has completed and flushed.
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait_prerequisites() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// An NVTX range over one host call (the library's entry points), for
+// Nsight timelines.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
 
 // Launch `kernel` so that it may start while the previous kernel on the
 // stream drains (programmatic stream serialization).  Every kernel launched

@@ -96,6 +96,7 @@ extern "C" int spec_verify_static(const void* logits, int logits_dtype, const in
                                   const int64_t* pos_base, int32_t* accepted_len_out,
                                   int32_t* out_tokens, float* p_draft_out, float* row_stats_out,
                                   int32_t* status, cudaStream_t stream) {
+  spec::NvtxRange range("spec_verify_static");
   const size_t need = spec_verify_workspace(B, K, V);
   if (need == 0) return SPEC_ERR_INVALID_ARG;
   if (need > (size_t)SPEC_STATIC_SCRATCH_BYTES) return SPEC_ERR_TOO_LARGE;
