@@ -50,7 +50,9 @@ constexpr int kMkRows = 128;        // MMA M: request rows (rows >= B are zero)
 constexpr int kMkTile = 128;        // MMA N: vocabulary rows of W2^T per tile
 constexpr int kMkAtomK = 64;        // bf16 along K per 128-byte swizzle atom
 constexpr int kMkAtomBytes = 128 * 128;  // one atom of 128 rows x 128 bytes
-constexpr int kMkEpiWarps = 8;      // two per TMEM lane quarter, taking alternate tiles
+constexpr int kMkEpiWarps = 8;      // kMkHalves per TMEM lane quarter, taking tiles in turn
+constexpr int kMkHalves = kMkEpiWarps / 4;  // epilogue warps per lane quarter
+constexpr int kMkParts = 2 * kMkHalves;     // partials per (request, bias CTA)
 constexpr int kMkSub = 64;          // sub-block: the columns of a tile one epilogue warp takes
 constexpr int kMkRace = kRaceBlock; // race block: four sub-blocks (the blocks of every draw)
 constexpr int kMkThreads = 32 * (2 + kMkEpiWarps);  // warp 0 TMA, warp 1 MMA, then the epilogue
@@ -79,7 +81,7 @@ struct MarkovLaunch {
   const int64_t* pos_base;
   const int32_t* x0;
   __nv_bfloat16* E;  // [128, r]: W1 at the previous drafts
-  MkPartial* part;   // [B][G][4]: per bias CTA, per epilogue half and column half
+  MkPartial* part;   // [B][G][kMkParts]: per bias CTA, per epilogue group and column half
   float2* sub;       // [B][nsub_pad]: per 64-column sub-block (max, sum relative to fl(max*c2)), tau > 0
   int nsub, nsub_pad;
   int G;
@@ -247,8 +249,8 @@ __global__ void __launch_bounds__(kMkThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ntiles = (p.V + kMkTile - 1) / kMkTile;
   const int T = ntiles > (int)blockIdx.x ? (ntiles - 1 - (int)blockIdx.x) / p.G + 1 : 0;  // tile t: blockIdx.x + t G
-  // Epilogue warps: TMEM lane quarter q = warp % 4, half eh = the tiles with
-  // t % 2 == eh.  With B <= 64 the operand's rows 64..127 repeat rows 0..63,
+  // Epilogue warps: TMEM lane quarter q = warp % 4, group eh = the tiles with
+  // t % kMkHalves == eh.  With B <= 64 the operand's rows 64..127 repeat rows 0..63,
   // so every request row sits in two quarters: quarters 0-1 take a tile's
   // columns 0..63 and quarters 2-3 its columns 64..127, and all four SM
   // sub-partitions share the epilogue.  With B > 64 a warp takes its 32 rows
@@ -361,17 +363,14 @@ __global__ void __launch_bounds__(kMkThreads, 1)
     ArgState g{-INFINITY, INT_MAX};
     int32_t flags = 0;
     bool aborted = false;
-    uint4 uw[16];
-    for (int t = eh; t < T; t += 2) {
-      const int slot = t & 3;
-      const int v0 = ((int)blockIdx.x + t * p.G) * kMkTile;
-      // the warp's columns of U (bf16), fetched before the accumulator wait.
-      // A lane reads 128 consecutive bytes of its own row in 16-byte loads;
-      // the loads allocate in L1, so each 32-byte sector crosses from L2 once.
+    // A lane reads 128 consecutive bytes of its own row of U in 16-byte
+    // loads (one 64-column sub-block); the loads allocate in L1, so each
+    // 32-byte sector crosses from L2 once.
+    uint4 uw[8];
+    auto load_u = [&](int vb) {
 #pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        if (h >= 8 * nblk) break;
-        const int v = v0 + kMkSub * blk0 + 8 * h;
+      for (int h = 0; h < 8; ++h) {
+        const int v = vb + 8 * h;
         if (valid && p.u_vec && v + 8 <= p.V) {
           uw[h] = __ldg(reinterpret_cast<const uint4*>(p.U + urow + v));
         } else {
@@ -383,9 +382,15 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           uw[h] = make_uint4(e[0] | e[1] << 16, e[2] | e[3] << 16, e[4] | e[5] << 16, e[6] | e[7] << 16);
         }
       }
+    };
+    for (int t = eh; t < T; t += kMkHalves) {
+      const int slot = t & 3;
+      const int v0 = ((int)blockIdx.x + t * p.G) * kMkTile;
+      // the warp's first sub-block of U, fetched before the accumulator wait
+      load_u(v0 + kMkSub * blk0);
       // the warp's next tile of U, into L2 while this one is processed
-      if (valid && t + 2 < T) {
-        const int vn = ((int)blockIdx.x + (t + 2) * p.G) * kMkTile + kMkSub * blk0;
+      if (valid && t + kMkHalves < T) {
+        const int vn = ((int)blockIdx.x + (t + kMkHalves) * p.G) * kMkTile + kMkSub * blk0;
         const int ve = min(vn + kMkSub * nblk, p.V) - 1;
         if (vn < p.V)
           for (int x = vn; x <= ve; x += 64) {
@@ -402,6 +407,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       for (int cb = 0; cb < nblk; ++cb) {
         const int bcol = kMkSub * (blk0 + cb);  // the sub-block's first column in the tile
         const int sb = (v0 + bcol) / kMkSub;
+        if (cb > 0) load_u(v0 + bcol);  // B > 64: the warp's second sub-block
         SoftState blk{-INFINITY, 0.0f};
 #pragma unroll
         for (int ch = 0; ch < kMkSub / 32; ++ch) {
@@ -410,7 +416,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
           float cmax = -INFINITY;
 #pragma unroll
           for (int k = 0; k < 32; ++k) {
-            const uint4& w4 = uw[(kMkSub * cb + 32 * ch + k) >> 3];
+            const uint4& w4 = uw[(32 * ch + k) >> 3];
             const int e = k & 7;
             const uint32_t word = e < 2 ? w4.x : e < 4 ? w4.y : e < 6 ? w4.z : w4.w;
             l[k] += (e & 1) ? bf16_hi(word) : bf16_lo(word);  // -inf past V (U reads -inf there, the bias is 0)
@@ -454,7 +460,7 @@ __global__ void __launch_bounds__(kMkThreads, 1)
       o.L = kGreedy ? g.v : 0.0f;
       o.idx = kGreedy ? g.idx : INT_MAX;
       o.flags = flags;
-      MkPartial* dstp = p.part + ((size_t)row * p.G + blockIdx.x) * 4 + 2 * eh;
+      MkPartial* dstp = p.part + ((size_t)row * p.G + blockIdx.x) * kMkParts + 2 * eh;
       dstp[col_half] = o;
       if (!dup) {  // this warp covered both column halves
         MkPartial none{};
@@ -523,12 +529,12 @@ __global__ void __launch_bounds__(kPickThreads, 1) markov_pick_kernel(const Mark
       sq[h] = q < nq && 16 * q + 2 * h < p.nsub ? __ldcg(subrow + 8 * q + h) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
   }
 
-  // ---- merge the 4G partials of the bias CTAs ----
+  // ---- merge the kMkParts * G partials of the bias CTAs ----
   {
     SoftState st{-INFINITY, 0.0f};
     ArgState g{-INFINITY, INT_MAX};
     int32_t f = 0;
-    const int n = 4 * p.G;
+    const int n = kMkParts * p.G;
     const uint4* src = reinterpret_cast<const uint4*>(p.part + (size_t)i * n);
     for (int c = threadIdx.x; c < n; c += kPickThreads) {
       const uint4 lo = __ldcg(src + 2 * c), hi = __ldcg(src + 2 * c + 1);
@@ -820,7 +826,7 @@ static MarkovGeometry markov_geometry(int B, int V, int r, int sms) {
   g.nsub_pad = (g.nsub + 15) / 16 * 16;
   g.e_off = 0;
   g.part_off = ((size_t)kMkRows * r * 2 + 255) / 256 * 256;
-  g.sub_off = g.part_off + ((size_t)sizeof(MkPartial) * B * 4 * g.G + 255) / 256 * 256;
+  g.sub_off = g.part_off + ((size_t)sizeof(MkPartial) * B * kMkParts * g.G + 255) / 256 * 256;
   g.bad_off = g.sub_off + ((size_t)sizeof(float2) * B * g.nsub_pad + 255) / 256 * 256;
   g.bytes = g.bad_off + ((size_t)4 * B + 255) / 256 * 256;
   return g;
