@@ -66,7 +66,13 @@ def test_alloc_workload_sweep_and_ratios():
     assert g["depth"][B // 2:].mean() > g["depth"][:B // 2].mean()
 
 
-@pytest.mark.parametrize("B,K", [(1, 0), (1, 5), (3, 4), (7, 7), (64, 16), (512, 15), (8192, 0)])
+# The one-CTA kernel's paths: padded runs merged (B * KP <= 1024, KP the next
+# power of two >= K: (7, 7), (64, 16), (32, 17), (4, 255) and (3, 200) with
+# two merge levels, (1024, 1) and (1000, 1) with ten, pad runs past B), the
+# bitonic network when the padded runs do not fit ((33, 17), (100, 10)); and
+# the large kernel ((512, 15), (8192, 0)).
+@pytest.mark.parametrize("B,K", [(1, 0), (1, 5), (3, 4), (7, 7), (64, 16), (32, 17), (4, 255), (3, 200),
+                                 (1024, 1), (1000, 1), (33, 17), (100, 10), (512, 15), (8192, 0)])
 def test_random_allocations(B, K):
     rng = np.random.default_rng(B * 100 + K)
     for trial in range(3):
