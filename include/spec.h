@@ -245,7 +245,7 @@ int spec_verify(const void* logits, int logits_dtype, const int32_t* row_offsets
  *   - Returns SPEC_ERR_TOO_LARGE, launching nothing, when
  *     spec_verify_workspace(B, K, V) exceeds SPEC_STATIC_SCRATCH_BYTES
  *     (4 MiB holds about 260,000 16-byte row-chunk partials; B=64, K=16,
- *     V=201088 needs spec_verify_workspace(64, 16, 201088) = 88,064
+ *     V=201088 needs spec_verify_workspace(64, 16, 201088) = 87,808
  *     bytes).
  *   - The first call on a device looks up the array's device address (once
  *     per device and CUDA context, with that device current); make that

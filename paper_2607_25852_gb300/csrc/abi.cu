@@ -187,7 +187,6 @@ int spec::verify_impl(const void* logits, int logits_dtype, const int32_t* row_o
   p.race_part = reinterpret_cast<spec::RacePartial*>(base + g.race_part_off);
   p.draft_view = reinterpret_cast<float2*>(base + g.view_off);
   p.counters = reinterpret_cast<uint32_t*>(base + g.counters_off);
-  p.req_count = p.counters + B;
   p.R_max = B * (K + 1);
   p.NC = g.NC;
   p.chunk = g.chunk;

@@ -195,7 +195,6 @@ struct VerifyLaunch {
   RacePartial* race_part; // [B * NCS]
   float2* draft_view;     // [R_max]: (logit, q) at each row's draft token (t > 0)
   uint32_t* counters;     // [B] sampling-pass arrivals per request
-  uint32_t* req_count;    // [B] streaming-pass arrivals per request
   int R_max;              // B * (K + 1)
   int NC;                 // vocabulary chunks per row, streaming pass
   int chunk;              // elements per chunk (multiple of 8)

@@ -4,25 +4,25 @@
 // the drafted tokens in one pass by rejection sampling; temperature 0 is the
 // longest argmax-matching prefix):
 //
-//   stream_rows_kernel  one CTA per (request, row, vocabulary chunk).  Streams
-//                       its chunk once with 16-byte loads and writes a 16-byte
-//                       partial: (max, sum of 2^(l*c2 - fl(max*c2))) at t > 0,
-//                       (max, lowest argmax) at t = 0.  This is the HBM-bound
-//                       pass: every retained logit is read once.  The last CTA
-//                       of a request to finish (arrival counter, no spinning)
-//                       merges the request's partials and runs its decision
-//                       chain: p_j(z_{j+1}) from the merged statistics and one
-//                       Philox draw per draft, the first rejection, the
-//                       committed prefix, the argmax token at t = 0, and at
-//                       t > 0 a record of what the sampling pass needs.
-//                       Decisions of early requests overlap the streaming of
-//                       later ones.
-//   sample_kernel       t > 0 only: one CTA per (request, vocabulary chunk) of
-//                       the single row that is sampled (the residual row at the
-//                       first rejection, else the bonus row), running the
-//                       exponential race y = argmin E_v / w_v.  The last CTA of
-//                       the request to finish merges the race partials and
-//                       writes y.
+//   stream_rows_kernel    one CTA per (request, row, vocabulary chunk).
+//                         Streams its chunk once with 16-byte loads and
+//                         writes a 16-byte partial: (max, sum of
+//                         2^(l*c2 - fl(max*c2))) at t > 0, (max, lowest
+//                         argmax) at t = 0, and at t > 0 the target logit and
+//                         q at the row's draft token if its chunk holds it.
+//                         This is the HBM-bound pass: every retained logit is
+//                         read once.
+//   sample_kernel         t > 0: one CTA per (request, vocabulary chunk) of
+//                         the single row that is sampled.  Each CTA first
+//                         runs the request's decision chain (merged row
+//                         statistics, p_j(z_{j+1}), one Philox uniform per
+//                         draft, the first rejection): the residual row at the
+//                         first rejection, else the bonus row, is sampled by
+//                         the exponential race y = argmin E_v / w_v.  The last
+//                         CTA of the request to finish merges the race
+//                         partials, draws inside the winning block and writes
+//                         the outputs.
+//   greedy_decide_kernel  t = 0: one warp per request, the argmax chain.
 //
 // Nothing waits on another CTA: cross-CTA combination goes through arrival
 // counters (the last to arrive does the merge) or the kernel boundary.
@@ -63,21 +63,20 @@ VerifyGeometry verify_geometry(int B, int K, int V) {
   g.row_part_off = 0;
   g.race_part_off = round_up((long long)sizeof(RowPartial) * R_max * nc, 256);
   g.view_off = g.race_part_off + round_up((long long)sizeof(RacePartial) * B * ncs, 256);
-  // zero region: sampling arrivals [B], then streaming arrivals [B]
+  // zero region: the sampling pass's arrivals [B]
   g.counters_off = g.view_off + round_up((long long)sizeof(float2) * R_max, 256);
-  g.bytes = g.counters_off + round_up(sizeof(uint32_t) * 2LL * B, 256);
+  g.bytes = g.counters_off + round_up(sizeof(uint32_t) * (long long)B, 256);
   return g;
 }
 
 // ---------------------------------------------------------------------------
-// Decision chain (the last streaming CTA of a request)
+// Decision chain (every sampling CTA at t > 0; greedy_decide_kernel at t = 0)
 // ---------------------------------------------------------------------------
 // One warp.  Merges the chunk partials of rows 0..n (a lane per row), loads
 // the target logit and the draft probability at each draft, and runs the
-// decision chain.  Only one warp of a CTA decides at a time (its shared arrays
-// are per CTA).
-// The decision arrays of a CTA (row statistics, drafts, p_j(z)), kept after
-// the decision for the outputs written later.
+// decision chain.  Only one warp of a CTA decides at a time: the decision
+// arrays (row statistics, drafts, p_j(z)) are per CTA, and are kept after the
+// decision for the outputs written later.
 __shared__ float sh_m[kMaxRows];
 __shared__ float sh_S[kMaxRows];
 __shared__ int32_t sh_g[kMaxRows];
@@ -163,37 +162,22 @@ __device__ __forceinline__ void decide_request(const VerifyLaunch& p, int i, Req
   bad = __any_sync(0xFFFFFFFFu, bad);
   __syncwarp();
   decide_chain<kGreedy>(p, i, rs, pre, decide_arrays(), lz, qz, bad, outputs, rec_dst);
-  if (kGreedy && lane == 0) p.req_count[i] = 0u;  // leave the workspace zeroed for the next call
   __syncwarp();
 }
 
 // End of one (request, row, chunk) item, all threads of the CTA: the CTA
-// reduction and the chunk partial (valid requests).  At t = 0 the CTA then
-// arrives on the request's counter, and the last CTA to arrive decides the
-// request.  At t > 0 the sampling kernel, which waits for this grid anyway,
-// decides each request from the complete partials, so a streaming CTA ends
-// with its partial and holds no SM slot for a round trip.
+// reduction and the chunk partial (valid requests).  The kernel after this
+// one, which waits for this grid anyway, decides each request from the
+// complete partials (the sampling kernel at t > 0, greedy_decide_kernel at
+// t = 0), so a streaming CTA ends with its partial and holds no SM slot for
+// a round trip.
 template <typename T, bool kGreedy>
-__device__ __forceinline__ void finish_item(const VerifyLaunch& p, RowAcc<T, kGreedy>& acc, int i, const ReqShape& rs,
+__device__ __forceinline__ void finish_item(const VerifyLaunch& p, RowAcc<T, kGreedy>& acc, const ReqShape& rs,
                                             long long r, int c) {
-  __shared__ int sh_last;
   if (rs.valid) {
     const RowPartial out = cta_reduce_partial<T, kGreedy>(acc, p.c2);
     if (threadIdx.x == 0) p.row_part[(size_t)r * p.NC + c] = out;
   }
-  if (!kGreedy) return;
-  // ---- arrival; the last CTA of the request decides it (warp 0) ----
-  DecidePre pre;
-  if (threadIdx.x < 32) pre = decide_prefetch(p, i);
-  if (threadIdx.x == 0) {
-    __threadfence();  // the partial above before the count
-    const uint32_t target = rs.valid ? (uint32_t)(rs.n + 1) * (uint32_t)p.NC : 1u;
-    sh_last = atomicAdd(p.req_count + i, 1u) == target - 1u;
-  }
-  consumer_sync();
-  if (!sh_last || threadIdx.x >= 32) return;
-  __threadfence();  // the other CTAs' partials after their counts
-  decide_request<T, kGreedy>(p, i, rs, pre, true, nullptr);
 }
 
 // Item of CTA blockIdx.x: (request i, row j, chunk c), request-major, so
@@ -214,7 +198,7 @@ __device__ __forceinline__ StreamItem stream_item(const VerifyLaunch& p) {
 // Streaming pass with 16-byte loads from global memory (any alignment: a
 // scalar head and tail around the aligned body).
 template <typename T, bool kGreedy>
-__global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const VerifyLaunch p) {
+__global__ void __launch_bounds__(kStreamThreads, kGreedy ? 4 : 0) stream_rows_kernel(const VerifyLaunch p) {
   const StreamItem it = stream_item(p);
   pdl_wait_prerequisites();  // row offsets and depths come from the allocator
   const ReqShape rs = request_shape(p, it.i);
@@ -240,7 +224,21 @@ __global__ void __launch_bounds__(kStreamThreads) stream_rows_kernel(const Verif
       p.draft_view[r] = make_float2(lz, qz);
     }
   }
-  finish_item<T, kGreedy>(p, acc, it.i, rs, r, it.c);
+  finish_item<T, kGreedy>(p, acc, rs, r, it.c);
+}
+
+// t = 0: each request's decision, one warp (one CTA) per request, once the
+// streaming kernel has written every row's (max, lowest argmax) partials.
+// The request's shape and drafts are the allocator's and the caller's, loaded
+// (through L2) while the streaming kernel drains.
+template <typename T>
+__global__ void __launch_bounds__(32) greedy_decide_kernel(const VerifyLaunch p) {
+  const int i = blockIdx.x;
+  const ReqShape rs = request_shape<VerifyLaunch, true>(p, i);
+  const DecidePre pre = decide_prefetch<VerifyLaunch, true, false>(p, i);
+  pdl_wait_prerequisites();  // the row partials of the streaming kernel
+  pdl_launch_dependents();   // the commit kernel waits for this grid in turn
+  decide_request<T, true>(p, i, rs, pre, true, nullptr);
 }
 
 template <typename T>
@@ -400,7 +398,11 @@ static cudaError_t launch_typed(const VerifyLaunch& p, cudaStream_t stream, cuda
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   if (ev_after) cudaEventRecord(ev_after, stream);
-  if (greedy) return cudaSuccess;
+  if (greedy) {
+    err = launch_after_previous(greedy_decide_kernel<T>, dim3((unsigned)p.B), dim3(32), 0, stream, p);
+    if (err != cudaSuccess) return err;
+    return cudaGetLastError();
+  }
   // The sampling CTAs are launched while the streaming kernel drains and
   // wait (griddepcontrol.wait) for its completion.
   err = launch_after_previous(sample_kernel<T>, dim3((unsigned)((long long)p.B * p.NCS)), dim3(kSampleThreads), 0,
