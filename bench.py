@@ -246,9 +246,10 @@ class Step:
                       row_offsets=self.row_off, status=self.status)
 
     def launches_per_step(self):
-        # allocate (1) + verify: streaming with decisions (1) and, at t > 0, the
-        # sampling pass (1) + commit (1 for B <= 256, else 2)
-        return 1 + (1 if self.wl.temperature == 0 else 2) + (1 if self.wl.B <= 256 else 2)
+        # allocate (1) + verify: the streaming pass, then the decisions (t = 0)
+        # or the sampling pass with the decisions (t > 0) (2) + commit (1 for
+        # B <= 256, else 2)
+        return 1 + 2 + (1 if self.wl.B <= 256 else 2)
 
 
 def algorithmic_bytes(wl, acc, rows=None):
