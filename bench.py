@@ -43,6 +43,24 @@ KERNEL_SAMPLES = 30  # event-bracketed launches of the streaming kernel, at leas
 FALLBACK_HBM_GBS = 6800.0
 
 
+class L2Flush:
+    """Evicts L2 between timed iterations: a write of twice the L2 size, then a
+    read of another buffer of that size, so that L2 is left holding clean lines
+    only.  (After the write alone, L2 is full of dirty lines, which the next
+    kernel would write back to HBM while it reads its own inputs.)"""
+
+    def __init__(self, device):
+        import torch
+        self.w = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=device)
+        self.r = torch.ones(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+        self.s = torch.empty((), dtype=torch.float32, device=device)
+
+    def __call__(self, k):
+        import torch
+        self.w.fill_(k & 0xFF)
+        torch.sum(self.r, 0, out=self.s)
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -444,11 +462,11 @@ def run_ours(args):
         for e in pair:
             e.record(stream)
     # A step whose inputs fit in L2 would find them cached from the step
-    # before: then L2 is flushed between steps (a write larger than L2) and
+    # before: then L2 is flushed between steps (L2Flush) and
     # only the steps themselves are timed.
     flush = None
     if alg["logits"] < 2 * L2_BYTES:
-        flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=device)
+        flush = L2Flush(device)
     torch.cuda.synchronize()
     barrier(dist)
     torch.cuda.synchronize()
@@ -462,7 +480,7 @@ def run_ours(args):
         start.record(stream)
         for k in range(args.steps):
             if flush is not None:
-                flush.fill_(k & 0xFF)
+                flush(k)
                 ev[k][0].record(stream)
             step.run()
             if flush is not None:
@@ -491,7 +509,7 @@ def run_ours(args):
         gpu_head_start(n_k)
         for k in range(n_k):
             if flush is not None:
-                flush.fill_(k & 0xFF)
+                flush(k)
             spec.spec_profile_stream_pass(kev[k][0], kev[k][1])
             step.run()
         torch.cuda.synchronize()
@@ -717,37 +735,55 @@ def run_sharded(args):
         torch.cuda.synchronize()
     round_ms = a.elapsed_time(b) / args.steps
 
-    # per-rank calls of shard 0, each bracketed by its own events
+    # Per-rank calls.  Each is timed (1) in a loop of back-to-back calls that
+    # cycles through the S shards, its mean per call: the stats and sample
+    # calls then read S x a shard's logits in turn, more than L2, so that no
+    # call finds its inputs in L2 (decide and finish read the records, which a
+    # rank receives from the all-gather just before); and (2) alone, after an
+    # L2 flush, the median of `steps` calls, which adds the latency of an
+    # isolated launch and the event clock's granularity (about 1 us).
     sb, rb = R * spec.SHARD_STAT_BYTES, B * spec.SHARD_RACE_BYTES
-    q0 = None if qs is None else qs[0]
+    sl = [slice(s * sb, (s + 1) * sb) for s in range(S)]
+    rl = [slice(s * rb, (s + 1) * rb) for s in range(S)]
+    qsh = (lambda s: None) if qs is None else (lambda s: qs[s])
     calls = {
-        "stats": lambda: spec.spec_shard_stats(lgs[0], wl.drafts, q0, B, K, V, 0, t, wl.pos_base,
-                                               rnd.stats[:sb], rnd.ws[0], status=status),
-        "decide": lambda: spec.spec_shard_decide(rnd.stats, S, wl.drafts, q0 is not None, B, K, V, t, wl.seeds,
-                                                 wl.request_ids, wl.pos_base, acc, tok,
-                                                 decisions_out=rnd.decisions, status=status),
-        "sample": lambda: spec.spec_shard_sample(lgs[0], q0, rnd.decisions, B, K, V, 0, t, wl.seeds,
-                                                 wl.request_ids, rnd.races[:rb], rnd.ws[0], status=status),
-        "finish": lambda: spec.spec_shard_finish(rnd.races, S, rnd.decisions, B, K, V, t, wl.seeds,
-                                                 wl.request_ids, acc, tok, status=status),
+        "stats": lambda s: spec.spec_shard_stats(lgs[s], wl.drafts, qsh(s), B, K, V, bounds[s], t, wl.pos_base,
+                                                 rnd.stats[sl[s]], rnd.ws[s], status=status),
+        "decide": lambda s: spec.spec_shard_decide(rnd.stats, S, wl.drafts, qs is not None, B, K, V, t, wl.seeds,
+                                                   wl.request_ids, wl.pos_base, acc, tok,
+                                                   decisions_out=rnd.decisions, status=status),
+        "sample": lambda s: spec.spec_shard_sample(lgs[s], qsh(s), rnd.decisions, B, K, V, bounds[s], t, wl.seeds,
+                                                   wl.request_ids, rnd.races[rl[s]], rnd.ws[s], status=status),
+        "finish": lambda s: spec.spec_shard_finish(rnd.races, S, rnd.decisions, B, K, V, t, wl.seeds,
+                                                   wl.request_ids, acc, tok, status=status),
     }
-    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=device)
-    per = {}
+    flush = L2Flush(device)
+    n_loop = 4 * S
+    per, alone = {}, {}
     for name, fn in calls.items():
         if t == 0 and name in ("sample", "finish"):
             continue
-        ts = []
+        ts, ts1 = [], []
         for k in range(args.steps):
             round_()                    # leaves every record of this round in place
-            flush.fill_(k & 0xFF)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            torch.cuda._sleep(200000)  # queue the launches ahead of the start event
-            e0.record(stream)
-            fn()
-            e1.record(stream)
             torch.cuda.synchronize()
-            ts.append(e0.elapsed_time(e1))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            gpu_head_start(1, host_us_per_step=40.0 * n_loop)  # queue the launches ahead of the start event
+            e0.record(stream)
+            for c in range(n_loop):
+                fn(c % S)
+            e1.record(stream)
+            flush(k)
+            e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(200000)
+            e2.record(stream)
+            fn(0)
+            e3.record(stream)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1) / n_loop)
+            ts1.append(e2.elapsed_time(e3))
         per[name] = 1e3 * statistics.median(ts)
+        alone[name] = 1e3 * statistics.median(ts1)
     assert int(status.item()) == 0
     peak, peak_kind = measured_peak()
     esize = 2 if wl.dtype == "bf16" else 4
@@ -764,12 +800,18 @@ def run_sharded(args):
                    "parallelism": f"vocabulary split into {S} shards, all on one GPU (records written "
                                   "side by side in place of the all-gathers)"},
         "per_rank_us": {k: round(v, 2) for k, v in per.items()},
+        "per_rank_us_how": (f"mean per call over {n_loop} back-to-back calls cycling through the {S} shards, "
+                            f"median of {args.steps} loops"),
+        "per_rank_alone_us": {k: round(v, 2) for k, v in alone.items()},
+        "per_rank_alone_us_how": "one call alone after an L2 flush (L2Flush), event-bracketed, median",
         "per_rank_critical_path_us": round(sum(per.values()), 2),
         "exchange_bytes_per_rank": {"stats": sb, "races": rb if t > 0 else 0},
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None, "kernel": "shard_stats_kernel",
                      "peak_kind": peak_kind, "algorithmic_bytes_per_launch": stats_bytes,
-                     "avg_launch_us": round(per["stats"], 2)},
+                     "avg_launch_us": round(per["stats"], 2),
+                     "alone": {"us": round(alone["stats"], 2),
+                               "frac": round(stats_bytes / (alone["stats"] * 1e-6) / 1e9 / peak, 4)}},
         "clocks": clocks.summary(),
         "gpu_launches": (2 * S + 2 if t > 0 else S + 1) * args.steps,
     }
@@ -807,13 +849,13 @@ def run_draft(args):
     nbytes = di.logits.numel() * di.logits.element_size()
     flush = None
     if nbytes < 2 * L2_BYTES:
-        flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=device)
+        flush = L2Flush(device)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     with ClockSampler(0) as clocks:
         gpu_head_start(args.steps)
         for k in range(args.steps):
             if flush is not None:
-                flush.fill_(k & 0xFF)
+                flush(k)
             ev[k][0].record(stream)
             step()
             ev[k][1].record(stream)

@@ -157,21 +157,19 @@ static ShardGeometry shard_geometry(int B, int K, int Vs) {
 // CTA of a row to finish merges the row's chunk partials into its record.
 // ---------------------------------------------------------------------------
 // The row's draft, seen from this shard: its logit and q value if the shard
-// owns the draft's column.  Loaded before the stream, used after it.
+// owns the draft's column.  The draft token is loaded before the stream, the
+// logit and q value after it (no dependent round trips ahead of the loads).
 struct DraftView {
   float lz, qz;
   int32_t owned;
 };
 template <typename T>
-__device__ __forceinline__ DraftView draft_view(const ShardLaunch& p, int i, int j, const ReqShape& rs, const T* row) {
+__device__ __forceinline__ DraftView draft_view(const ShardLaunch& p, int i, int j, int z, const T* row) {
   DraftView d{0.0f, 1.0f, 0};
-  if (j < rs.n) {
-    const int z = __ldg(p.drafts + (size_t)i * p.K + j);
-    if (z >= p.v_begin && z < p.v_begin + p.Vs) {
-      d.owned = 1;
-      d.lz = load_elem(row + (z - p.v_begin));
-      if (p.dense_q) d.qz = load_any(p.q, p.q_dtype, ((int64_t)i * p.K + j) * (int64_t)p.Vs + (z - p.v_begin));
-    }
+  if (z >= p.v_begin && z < p.v_begin + p.Vs) {
+    d.owned = 1;
+    d.lz = load_elem(row + (z - p.v_begin));
+    if (p.dense_q) d.qz = load_any(p.q, p.q_dtype, ((int64_t)i * p.K + j) * (int64_t)p.Vs + (z - p.v_begin));
   }
   return d;
 }
@@ -190,8 +188,10 @@ __device__ __forceinline__ void write_stat(const ShardLaunch& p, long long r, fl
   p.stats[r] = st;
 }
 
-template <typename T, bool kGreedy>
-__global__ void __launch_bounds__(kStreamThreads) shard_stats_kernel(const ShardLaunch p) {
+// kThreads = 256 (four CTAs per SM) or 128 (eight per SM): the same threads
+// and loads in flight per SM either way.
+template <typename T, bool kGreedy, int kThreads>
+__global__ void __launch_bounds__(kThreads, 1024 / kThreads) shard_stats_kernel(const ShardLaunch p) {
   const int per_req = (p.K + 1) * p.NC;
   const int i = blockIdx.x / per_req;
   const int rem = blockIdx.x - i * per_req;
@@ -203,12 +203,14 @@ __global__ void __launch_bounds__(kStreamThreads) shard_stats_kernel(const Shard
   pdl_launch_dependents();
   const long long r = rs.row0 + j;
   const T* row = static_cast<const T*>(p.logits) + (size_t)r * (size_t)p.Vs;
-  DraftView dv{0.0f, 1.0f, 0};
-  if (threadIdx.x == 0) dv = draft_view(p, i, j, rs, row);
+  // the row's draft (thread 0; -1 past the request's depth)
+  const int z = threadIdx.x == 0 && j < rs.n ? __ldg(p.drafts + (size_t)i * p.K + j) : -1;
   RowAcc<T, kGreedy> acc;
   const int v0 = c * p.chunk;
-  stream_chunk<T, kGreedy>(acc, row, v0, min(p.Vs, v0 + p.chunk), p.v_begin, p.c2);
-  const RowPartial part = cta_reduce_partial<T, kGreedy>(acc, p.c2);
+  stream_chunk<T, kGreedy, kThreads, kUnroll, true>(acc, row, v0, min(p.Vs, v0 + p.chunk), p.v_begin, p.c2);
+  DraftView dv{0.0f, 1.0f, 0};
+  if (threadIdx.x == 0) dv = draft_view(p, i, j, z, row);
+  const RowPartial part = cta_reduce_partial<T, kGreedy, kThreads>(acc, p.c2);
   if (p.NC == 1) {  // the whole shard row in this CTA: its partial is the record
     if (threadIdx.x == 0) write_stat(p, r, part.m, part.s, kGreedy ? part.idx : INT_MAX, part.flags, dv);
     return;
@@ -263,6 +265,12 @@ __global__ void __launch_bounds__(kStreamThreads) shard_stats_kernel(const Shard
     write_stat(p, r, st.m, st.s, st.idx, st.flags, dv);
     p.row_count[r] = 0u;  // leave the workspace zeroed for the next call
   }
+}
+
+template <typename T, bool kGreedy>
+static cudaError_t launch_stats(unsigned grid, bool narrow, cudaStream_t stream, const ShardLaunch& p) {
+  return narrow ? launch_after_previous(shard_stats_kernel<T, kGreedy, 128>, dim3(grid), dim3(128), 0, stream, p)
+                : launch_after_previous(shard_stats_kernel<T, kGreedy, 256>, dim3(grid), dim3(256), 0, stream, p);
 }
 
 // ---------------------------------------------------------------------------
@@ -774,17 +782,21 @@ extern "C" int spec_shard_stats(const void* logits_shard, int logits_dtype, cons
   p.NC = g.NC;
   p.chunk = g.chunk;
   const unsigned grid = (unsigned)((long long)B * (K + 1) * p.NC);
-  const dim3 block(spec::kStreamThreads);
+  // 256-thread CTAs while the grid fits in one wave of them (four per SM),
+  // else 128-thread CTAs (eight per SM), which take twice the rows into the
+  // first wave
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return SPEC_ERR_CUDA;
+  const bool narrow = (long long)grid > 4LL * sms;
   const bool greedy = temperature == 0.0f;
   cudaError_t err;
   if (logits_dtype == SPEC_F32)
-    err = greedy ? spec::launch_after_previous(spec::shard_stats_kernel<float, true>, dim3(grid), block, 0, stream, p)
-                 : spec::launch_after_previous(spec::shard_stats_kernel<float, false>, dim3(grid), block, 0, stream, p);
+    err = greedy ? spec::launch_stats<float, true>(grid, narrow, stream, p)
+                 : spec::launch_stats<float, false>(grid, narrow, stream, p);
   else
-    err = greedy ? spec::launch_after_previous(spec::shard_stats_kernel<__nv_bfloat16, true>, dim3(grid), block, 0,
-                                               stream, p)
-                 : spec::launch_after_previous(spec::shard_stats_kernel<__nv_bfloat16, false>, dim3(grid), block, 0,
-                                               stream, p);
+    err = greedy ? spec::launch_stats<__nv_bfloat16, true>(grid, narrow, stream, p)
+                 : spec::launch_stats<__nv_bfloat16, false>(grid, narrow, stream, p);
   if (err != cudaSuccess || cudaGetLastError() != cudaSuccess) return SPEC_ERR_CUDA;
   return SPEC_OK;
 }

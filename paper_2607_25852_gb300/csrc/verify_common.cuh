@@ -58,9 +58,10 @@ __device__ __forceinline__ bool key_better(KeyState a, KeyState b) {
   return a.key < b.key || (a.key == b.key && a.idx < b.idx);
 }
 
-// Barrier over the kStreamThreads threads of a streaming CTA.
+// Barrier over the kThreads threads of a streaming CTA.
+template <int kThreads = kStreamThreads>
 __device__ __forceinline__ void consumer_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kStreamThreads) : "memory");
+  asm volatile("bar.sync 1, %0;" ::"n"(kThreads) : "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -150,7 +151,9 @@ struct RowAcc {
 
   // kN 16-byte vectors; vector u holds entries v_of[u] .., v_of[u] ==
   // INT_MAX marks a padding vector (-inf entries), which adds nothing.
-  template <int kN>
+  // kAnyOrder: the thread's vectors may come in any order of their indices
+  // (t = 0 then compares indices at a tie), else in increasing order.
+  template <int kN, bool kAnyOrder = false>
   __device__ __forceinline__ void tile(const uint4 (&w)[kN], const int (&v_of)[kN], float c2) {
     using VT = Vec<T>;
     constexpr int VEC = VT::N;
@@ -170,7 +173,8 @@ struct RowAcc {
       // first vector that reaches the maximum
 #pragma unroll
       for (int u = 0; u < kN; ++u) {
-        if (v_of[u] != INT_MAX && (g.idx == INT_MAX || wm[u] > g.v)) {
+        const bool earlier_tie = kAnyOrder && wm[u] == g.v && v_of[u] < (g_v0 != INT_MAX ? g_v0 : g.idx);
+        if (v_of[u] != INT_MAX && (g.idx == INT_MAX || wm[u] > g.v || earlier_tie)) {
           g.v = wm[u];
           g_word = w[u];
           g_v0 = v_of[u];
@@ -205,11 +209,15 @@ struct RowAcc {
   }
 };
 
-// Streams entries [v0, v1) of `row` into acc with 16-byte loads, kUnroll
-// vectors in flight per thread (any alignment: a scalar head and tail around
-// the aligned body).  Indices reported to acc are v + vofs (a shard's first
-// column, or 0).
-template <typename T, bool kGreedy>
+// Streams entries [v0, v1) of `row` into acc with 16-byte loads, kN vectors
+// in flight per thread of the kThreads of the CTA (any alignment: a scalar
+// head and tail around the aligned body).  Indices reported to acc are
+// v + vofs (a shard's first column, or 0).
+//
+// kFold: vectors past the last whole round, if at most one per thread, are
+// loaded with the first round (a ninth vector for some threads) instead of
+// making a round trip of their own at the end.
+template <typename T, bool kGreedy, int kThreads = kStreamThreads, int kN = kUnroll, bool kFold = false>
 __device__ __forceinline__ void stream_chunk(RowAcc<T, kGreedy>& acc, const T* row, int v0, int v1, int vofs,
                                              float c2) {
   using VT = Vec<T>;
@@ -223,29 +231,43 @@ __device__ __forceinline__ void stream_chunk(RowAcc<T, kGreedy>& acc, const T* r
   if ((int)threadIdx.x < head) acc.scalar(vofs + v0 + threadIdx.x, load_elem(row + v0 + threadIdx.x), c2);
   // body: 16-byte vectors
   const uint4* vp = reinterpret_cast<const uint4*>(row + body0);
-  for (int base = threadIdx.x; base < nvec; base += kStreamThreads * kUnroll) {
-    uint4 w[kUnroll];
-    int v_of[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int vi = base + u * kStreamThreads;
-      w[u] = vi < nvec ? ldg_stream(vp + vi) : make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad);
-      v_of[u] = vi < nvec ? vofs + body0 + vi * VEC : INT_MAX;
+  int nround = nvec;  // vectors taken in whole-round steps
+  uint4 xw[1] = {make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad)};
+  int xv[1] = {INT_MAX};
+  if (kFold) {
+    const int rem = nvec % (kThreads * kN);
+    if (rem != 0 && rem <= kThreads && nvec > rem) {
+      nround = nvec - rem;
+      if ((int)threadIdx.x < rem) {
+        xw[0] = ldg_stream(vp + nround + threadIdx.x);
+        xv[0] = vofs + body0 + (nround + threadIdx.x) * VEC;
+      }
     }
-    acc.template tile<kUnroll>(w, v_of, c2);
+  }
+  for (int base = threadIdx.x; base < nround; base += kThreads * kN) {
+    uint4 w[kN];
+    int v_of[kN];
+#pragma unroll
+    for (int u = 0; u < kN; ++u) {
+      const int vi = base + u * kThreads;
+      w[u] = vi < nround ? ldg_stream(vp + vi) : make_uint4(VT::kPad, VT::kPad, VT::kPad, VT::kPad);
+      v_of[u] = vi < nround ? vofs + body0 + vi * VEC : INT_MAX;
+    }
+    acc.template tile<kN, kFold>(w, v_of, c2);
+    if (kFold && base == (int)threadIdx.x) acc.template tile<1, true>(xw, xv, c2);
   }
   // tail: the last < VEC elements (highest indices)
   if (tail0 + (int)threadIdx.x < v1) acc.scalar(vofs + tail0 + threadIdx.x, load_elem(row + tail0 + threadIdx.x), c2);
 }
 
-// The CTA's (kStreamThreads threads) reduction of a streamed chunk into one
+// The CTA's (kThreads threads) reduction of a streamed chunk into one
 // partial, valid in thread 0.  Every thread of the CTA calls it.
-template <typename T, bool kGreedy>
+template <typename T, bool kGreedy, int kThreads = kStreamThreads>
 __device__ __forceinline__ RowPartial cta_reduce_partial(RowAcc<T, kGreedy>& acc, float c2) {
-  __shared__ float sh_a[kStreamThreads / 32];
-  __shared__ float sh_b[kStreamThreads / 32];
-  __shared__ int32_t sh_i[kStreamThreads / 32];
-  __shared__ int32_t sh_f[kStreamThreads / 32];
+  __shared__ float sh_a[kThreads / 32];
+  __shared__ float sh_b[kThreads / 32];
+  __shared__ int32_t sh_i[kThreads / 32];
+  __shared__ int32_t sh_f[kThreads / 32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   acc.finalize();
   const int32_t flags = __reduce_or_sync(0xFFFFFFFFu, (unsigned)acc.flags);
@@ -262,11 +284,11 @@ __device__ __forceinline__ RowPartial cta_reduce_partial(RowAcc<T, kGreedy>& acc
       sh_i[warp] = g.idx;
       sh_f[warp] = flags;
     }
-    consumer_sync();
+    consumer_sync<kThreads>();
     if (threadIdx.x == 0) {
       ArgState best{sh_a[0], sh_i[0]};
       int32_t f = sh_f[0];
-      for (int k = 1; k < kStreamThreads / 32; ++k) {
+      for (int k = 1; k < kThreads / 32; ++k) {
         ArgState o{sh_a[k], sh_i[k]};
         if (arg_better(o, best)) best = o;
         f |= sh_f[k];
@@ -287,11 +309,11 @@ __device__ __forceinline__ RowPartial cta_reduce_partial(RowAcc<T, kGreedy>& acc
       sh_b[warp] = st.s;
       sh_f[warp] = flags;
     }
-    consumer_sync();
+    consumer_sync<kThreads>();
     if (threadIdx.x == 0) {
       SoftState all{sh_a[0], sh_b[0]};
       int32_t f = sh_f[0];
-      for (int k = 1; k < kStreamThreads / 32; ++k) {
+      for (int k = 1; k < kThreads / 32; ++k) {
         all = soft_merge(all, SoftState{sh_a[k], sh_b[k]}, c2);
         f |= sh_f[k];
       }

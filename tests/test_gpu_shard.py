@@ -63,6 +63,37 @@ def test_sampled_matches_oracle(layout, dtype, qmode):
     _check(wl, 0.7, LAYOUTS[layout](wl.V))
 
 
+@pytest.mark.parametrize("t", [0.0, 0.7])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_more_rows_than_one_wave_of_wide_stats_ctas(t, dtype):
+    """Past four stats CTAs per SM (one CTA per row here: K = 3, B = SMs + 8,
+    V_s < 16384), spec_shard_stats streams with 128-thread CTAs instead of
+    256-thread ones; the result does not depend on which."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    wl = _random_case(12345, dtype, t, "dense", B=sms + 8, K=3, seed=24)
+    gpu, _, _ = _check(wl, t, LAYOUTS["ragged3"](wl.V))
+    if t == 0.0:
+        _same_as_unsharded(wl, gpu)
+
+
+@pytest.mark.parametrize("t", [0.0, 0.7])
+@pytest.mark.parametrize("narrow", [False, True])
+def test_stats_rows_with_a_short_last_round(t, narrow):
+    """Shard rows whose 16-byte vectors run past whole load rounds by at most
+    one per thread (2048 + 100 vectors with 256-thread stats CTAs, 1024 + 50
+    with 128-thread ones): the remainder is loaded with the first round.
+    Logits rounded to integers tie the maximum in many places; at t = 0 the
+    lowest index must still win."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    B, K = (sms + 8, 3) if narrow else (5, 4)
+    Vs = 8 * (1024 + 50) if narrow else 8 * (2048 + 100)
+    wl = _random_case(Vs + 3000, "bf16", t, "dense", B=B, K=K, seed=25)
+    wl.logits = wl.logits.float().round().to(wl.logits.dtype)
+    gpu, _, _ = _check(wl, t, [0, Vs, wl.V])
+    if t == 0.0:
+        _same_as_unsharded(wl, gpu)
+
+
 @pytest.mark.parametrize("t", [0.0, 1.0])
 def test_shards_inside_one_race_block(t):
     """V = 1000 (four race blocks, the last one partial): a shard that lies
