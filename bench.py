@@ -853,6 +853,19 @@ def run_draft(args):
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     with ClockSampler(0) as clocks:
         gpu_head_start(args.steps)
+        if flush is None:
+            # steps back to back, as a drafter runs them (an event between two
+            # launches would keep the next from launching while the last drains)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for k in range(args.steps):
+                step()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ms_per_step = a.elapsed_time(b) / args.steps
+        # single steps, each bracketed by events: their spread (and the time
+        # itself where an L2 flush has to stay out of it)
+        gpu_head_start(args.steps)
         for k in range(args.steps):
             if flush is not None:
                 flush(k)
@@ -861,7 +874,8 @@ def run_draft(args):
             ev[k][1].record(stream)
         torch.cuda.synchronize()
     ms = [a.elapsed_time(b) for a, b in ev]
-    ms_per_step = statistics.mean(ms)
+    if flush is not None:
+        ms_per_step = statistics.mean(ms)
     peak, peak_kind = measured_peak()
     achieved = nbytes / (ms_per_step * 1e-3) / 1e9
     line = {
@@ -875,6 +889,9 @@ def run_draft(args):
                      "peak_kind": peak_kind, "algorithmic_bytes_per_launch": nbytes,
                      "avg_launch_us": round(1e3 * ms_per_step, 2)},
         "step_ms_p10_p50_p90": [float(np.percentile(ms, q)) for q in (10, 50, 90)],
+        "step_ms_how": "single steps, each bracketed by events (no overlap with the step before)",
+        "ms_per_step_how": ("steps back to back between two events" if flush is None
+                            else "mean of single steps bracketed by events, L2 flushed between them"),
         "mean_confidence": float(c.mean().item()),
         "clocks": clocks.summary(),
         "gpu_launches": args.steps,
@@ -918,13 +935,23 @@ def run_markov(args):
     assert int(status.item()) == 0, "device reported an error"
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     with ClockSampler(0) as clocks:
+        # steps back to back (each step's 2K + 1 launches chained as always)
+        gpu_head_start(args.steps, host_us_per_step=200.0)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for k in range(args.steps):
+            step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / args.steps
+        # single steps, each bracketed by events: their spread
         gpu_head_start(args.steps, host_us_per_step=200.0)
         for k in range(args.steps):
             ev[k][0].record(stream)
             step()
             ev[k][1].record(stream)
         torch.cuda.synchronize()
-    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    ms1 = [a.elapsed_time(b) for a, b in ev]
     peak, peak_kind = measured_peak()
     # per position: the whole W2 (V x r) and the position's base logits (B x V)
     per_pos = V * r * 2 + B * V * 2
@@ -942,6 +969,9 @@ def run_markov(args):
                      "avg_step_us": round(ms * 1e3, 2)},
         "tensor_tflops": round(flops / (ms * 1e-3) / 1e12, 2),
         "per_position_us": round(ms * 1e3 / K, 2),
+        "ms_per_step_how": "steps back to back between two events",
+        "step_ms_p10_p50_p90": [float(np.percentile(ms1, q)) for q in (10, 50, 90)],
+        "step_ms_how": "single steps, each bracketed by events (no overlap with the step before)",
         "clocks": clocks.summary(),
         "gpu_launches": (1 + 2 * K) * args.steps,
     }

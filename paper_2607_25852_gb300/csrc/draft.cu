@@ -244,17 +244,27 @@ __device__ __forceinline__ SoftState soft_merge_fast(SoftState a, SoftState b, f
   return a;
 }
 
+// The level-1 race words of blocks g0 .. g0+31 (g0 a multiple of 32), lane
+// l holding block g0 + l's: word l & 3 of the Philox quad at counter
+// (g0 >> 2) + (l >> 2).  One quad per lane serves 32 / N rounds.
+__device__ __forceinline__ uint32_t race_words(int g0, int lane, uint32_t position, uint64_t req, uint32_t k0,
+                                               uint32_t k1) {
+  const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)((g0 >> 2) + (lane >> 2))), k0, k1);
+  const int e = lane & 3;
+  return e == 0 ? rq.x : e == 1 ? rq.y : e == 2 ? rq.z : rq.w;
+}
+
 // One round of N consecutive race blocks b0 .. b0+N-1 of the warp (blocks at
 // or past b_hi were loaded as -inf).  Every value is taken relative to the
 // round's max M_r: the blocks' sums of 2^(l*c2 - fl(M_r*c2)) (a block whose
 // weight underflows against M_r is more than 2^-126 below the round's best
 // and cannot win the race), the round's softmax contribution, and each
 // block's level-1 candidate (L = log2 E_b - log2 sum_b, M = M_r), one block
-// per lane group.
+// per lane group.  Lane l's `rword` is the race word of block g0 + l, g0 the
+// first block of the group of 32 that holds this round (race_words).
 template <typename T, bool kGreedy>
 __device__ __forceinline__ void draft_round(WarpDraftState& ws, const uint4 (&w)[Lane8<T>::kBlocksPerRound][Lane8<T>::kWords],
-                                            int b0, int b_hi, int lane, float c2, uint32_t position, uint64_t req,
-                                            uint32_t k0, uint32_t k1) {
+                                            int b0, int b_hi, int lane, float c2, uint32_t rword) {
   using L8 = Lane8<T>;
   constexpr int N = L8::kBlocksPerRound;
   // ---- the round's max (+inf makes the row unusable; a NaN is caught by
@@ -321,8 +331,7 @@ __device__ __forceinline__ void draft_round(WarpDraftState& ws, const uint4 (&w)
   if (kGreedy) return;
   // ---- level-1 candidates, one block per lane group ----
   const int b = b0 + ub;
-  const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)(b >> 2)), k0, k1);
-  const uint32_t word = (b & 3) == 0 ? rq.x : (b & 3) == 1 ? rq.y : (b & 3) == 2 ? rq.z : rq.w;
+  const uint32_t word = __shfl_sync(0xFFFFFFFFu, rword, b & 31);
   // E near 0 needs log1pf; log2 of E and of the sum go to lg2.approx, whose
   // absolute error (~1e-7) is what a log-domain key can afford
   KeyState cand{INFINITY, INT_MAX};
@@ -389,9 +398,11 @@ __global__ void __launch_bounds__(kDraftThreads, 4) draft_rows_kernel(const Draf
   const uint64_t seed = __ldg(reinterpret_cast<const unsigned long long*>(p.seeds) + i);
   const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
   WarpDraftState ws;
+  uint32_t rword = 0;
   for (int b0 = b_lo; b0 < b_hi; b0 += kBPR) {
     if (b0 != b_lo) load_round(b0);
-    draft_round<T, kGreedy>(ws, w, b0, b_hi, lane, p.c2, position, req, k0, k1);
+    if (!kGreedy && (b0 == b_lo || (b0 & 31) == 0)) rword = race_words(b0 & ~31, lane, position, req, k0, k1);
+    draft_round<T, kGreedy>(ws, w, b0, b_hi, lane, p.c2, rword);
   }
 
   // ---- the segment's partial; the last warp of the row goes on ----
