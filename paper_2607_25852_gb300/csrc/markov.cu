@@ -514,19 +514,23 @@ __global__ void __launch_bounds__(kPickThreads, 1) markov_pick_kernel(const Mark
   // W2^T tiles and waits for this grid before it reads E
   pdl_launch_dependents();
   pdl_wait_prerequisites();
-  if (threadIdx.x < p.r) sh_e[threadIdx.x] = p.E[(size_t)i * p.r + threadIdx.x];
+  // this position's operand row, kept in a register until level 2 (a store
+  // to shared memory now would hold the thread's next loads back a round trip)
+  const __nv_bfloat16 e_own = (int)threadIdx.x < p.r ? p.E[(size_t)i * p.r + threadIdx.x] : __float2bfloat16(0.0f);
 
-  // ---- tau > 0: this thread's first quad of race blocks (16 sub-blocks),
-  // loaded together with the partials below ----
+  // a bad request stays bad: the flag of the positions before, read now
+  const uint32_t was_bad = threadIdx.x == 0 ? __ldcg(p.req_bad + i) : 0u;
+
+  // ---- tau > 0: this thread's first race block (four 64-column
+  // sub-blocks, two 16-byte loads), loaded together with the partials below ----
   const int nb = (p.V + kMkRace - 1) / kMkRace;  // race blocks
-  const int nq = (nb + 3) / 4;                     // quads (one Philox call each)
   const float4* subrow = reinterpret_cast<const float4*>(p.sub + (size_t)i * p.nsub_pad);
-  float4 sq[8];
+  const float4 kNoSub = make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+  float4 sq0 = kNoSub, sq1 = kNoSub;
   if (!kGreedy) {
-    const int q = threadIdx.x;
-#pragma unroll
-    for (int h = 0; h < 8; ++h)
-      sq[h] = q < nq && 16 * q + 2 * h < p.nsub ? __ldcg(subrow + 8 * q + h) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+    const int b = threadIdx.x;
+    if (b < nb) sq0 = __ldcg(subrow + 2 * b);
+    if (b < nb && 4 * b + 2 < p.nsub) sq1 = __ldcg(subrow + 2 * b + 1);
   }
 
   // ---- merge the kMkParts * G partials of the bias CTAs ----
@@ -549,8 +553,10 @@ __global__ void __launch_bounds__(kPickThreads, 1) markov_pick_kernel(const Mark
     for (int o = 16; o > 0; o >>= 1) {
       st = soft_merge(st, SoftState{__shfl_xor_sync(0xFFFFFFFFu, st.m, o), __shfl_xor_sync(0xFFFFFFFFu, st.s, o)},
                       p.c2);
-      const ArgState og{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
-      if (arg_better(og, g)) g = og;
+      if (kGreedy) {
+        const ArgState og{__shfl_xor_sync(0xFFFFFFFFu, g.v, o), __shfl_xor_sync(0xFFFFFFFFu, g.idx, o)};
+        if (arg_better(og, g)) g = og;
+      }
     }
     f = (int32_t)__reduce_or_sync(0xFFFFFFFFu, (unsigned)f);
     if (lane == 0) {
@@ -565,40 +571,35 @@ __global__ void __launch_bounds__(kPickThreads, 1) markov_pick_kernel(const Mark
   }
 
   // ---- level 1 (tau > 0): the key of every 256-entry block from its four
-  // 64-column sub-blocks, log2 E_b - log2 sum_b against the block's max ----
+  // 64-column sub-blocks, log2 E_b - log2 sum_b against the block's max; a
+  // block per thread ----
   if (!kGreedy) {
     MkKey best{INFINITY, 0.0f, INT_MAX};
-    for (int q = threadIdx.x; q < nq; q += kPickThreads) {
-      if (q != (int)threadIdx.x) {  // quads past the first: loaded here
-#pragma unroll
-        for (int h = 0; h < 8; ++h)
-          sq[h] = 16 * q + 2 * h < p.nsub ? __ldcg(subrow + 8 * q + h) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+    for (int b = threadIdx.x; b < nb; b += kPickThreads) {
+      if (b != (int)threadIdx.x) {  // blocks past the first: loaded here
+        sq0 = __ldcg(subrow + 2 * b);
+        sq1 = 4 * b + 2 < p.nsub ? __ldcg(subrow + 2 * b + 1) : kNoSub;
       }
-      const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)q), (uint32_t)seed,
+      const uint4 rq = philox(draw_counter(position, req, SPEC_PURPOSE_DRAFT, (uint32_t)(b >> 2)), (uint32_t)seed,
                               (uint32_t)(seed >> 32));
-      const uint32_t words[4] = {rq.x, rq.y, rq.z, rq.w};
-#pragma unroll
-      for (int s4 = 0; s4 < 4; ++s4) {
-        const int b = 4 * q + s4;
-        SoftState blk{-INFINITY, 0.0f};
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const float4 v = sq[2 * s4 + h];
-          // a sub-block past V reads (-inf, 0); a partial sub-block with 16 * q + 2 * h + 1 >= nsub was
-          // loaded whole but its second half is past the row's last sub-block
-          blk = mk_merge(blk, SoftState{v.x, v.y}, p.c2);
-          if (16 * q + 4 * s4 + 2 * h + 1 < p.nsub) blk = mk_merge(blk, SoftState{v.z, v.w}, p.c2);
-        }
-        if (b < nb && blk.m > -INFINITY && blk.s > 0.0f && isfinite(blk.s)) {
-          const float E = -log1pf(-((float)race_m(words[s4]) * 0x1p-24f));
-          const MkKey cand{mk_lg2(E) - mk_lg2(blk.s), blk.m, b};
-          if (mk_better(cand, best, p.c2)) best = cand;
-        }
+      const int e = b & 3;
+      const uint32_t word = e == 0 ? rq.x : e == 1 ? rq.y : e == 2 ? rq.z : rq.w;
+      // sub-blocks 4b .. 4b+3 in order; those at or past nsub add nothing
+      SoftState blk{-INFINITY, 0.0f};
+      blk = mk_merge(blk, SoftState{sq0.x, sq0.y}, p.c2);
+      if (4 * b + 1 < p.nsub) blk = mk_merge(blk, SoftState{sq0.z, sq0.w}, p.c2);
+      if (4 * b + 2 < p.nsub) blk = mk_merge(blk, SoftState{sq1.x, sq1.y}, p.c2);
+      if (4 * b + 3 < p.nsub) blk = mk_merge(blk, SoftState{sq1.z, sq1.w}, p.c2);
+      if (blk.m > -INFINITY && blk.s > 0.0f && isfinite(blk.s)) {
+        const float E = -log1pf(-((float)race_m(word) * 0x1p-24f));
+        const MkKey cand{mk_lg2(E) - mk_lg2(blk.s), blk.m, b};
+        if (mk_better(cand, best, p.c2)) best = cand;
       }
     }
     best = mk_warp_best(best, p.c2);
     if (lane == 0) sh_key[warp] = best;
   }
+  if ((int)threadIdx.x < p.r) sh_e[threadIdx.x] = e_own;
   __syncthreads();
   if (threadIdx.x < 32) {
     // warp 0 merges the warps' results
@@ -626,7 +627,7 @@ __global__ void __launch_bounds__(kPickThreads, 1) markov_pick_kernel(const Mark
       sh_m = st.m;
       sh_S = st.s;
       sh_idx = kGreedy ? g.idx : best.idx;
-      sh_bad = (f || p.req_bad[i] || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
+      sh_bad = (f || was_bad || !(st.m > -INFINITY) || !(st.s > 0.0f) || !isfinite(st.s) || sh_idx == INT_MAX)
                    ? 1 : 0;
     }
   }
