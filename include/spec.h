@@ -518,6 +518,19 @@ int spec_pack_rows(const void* src, size_t row_bytes, int B, int K, const int32_
  * ---------------------------------------------------------------------- */
 int spec_profile_stream_pass(cudaEvent_t before, cudaEvent_t after);
 
+/* ------------------------------------------------------------------------
+ * spec_check_bounded_wait -- failure-detection check of the library's
+ * bounded device waits (the mbarrier waits of spec_markov_draft's
+ * tensor-core pipeline).  Launches one warp that waits on an mbarrier no
+ * one arrives at: the wait gives up after about a second, sets
+ * SPEC_ERR_TIMEOUT in *status (first error wins) and the kernel returns, so
+ * the context stays usable.
+ *   status          device int32 [1].
+ * Returns SPEC_ERR_INVALID_ARG for a NULL status, SPEC_ERR_CUDA if the
+ * launch fails, else SPEC_OK (the timeout arrives through *status).
+ * ---------------------------------------------------------------------- */
+int spec_check_bounded_wait(int32_t* status, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

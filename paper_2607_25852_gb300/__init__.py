@@ -42,7 +42,7 @@ __all__ = [
     "spec_shard_finish", "shard_workspace", "spec_draft_workspace", "spec_draft", "draft_workspace",
     "spec_graph_begin_capture", "spec_graph_end_capture", "spec_graph_launch", "spec_graph_destroy",
     "spec_select_round", "spec_pack_rows", "spec_markov_workspace", "spec_markov_draft", "markov_workspace",
-    "spec_pointer_device_readable",
+    "spec_pointer_device_readable", "spec_check_bounded_wait",
 ]
 
 
@@ -335,6 +335,12 @@ def spec_shard_finish(races, S, decisions, B, K, V, temperature, seeds, request_
         _ptr(races), S, _ptr(decisions), B, K, V, float(temperature), _ptr(seeds), _ptr(request_ids),
         _ptr(accepted_len_out), _ptr(out_tokens), _ptr(status), _stream(stream))
     _check(code, "spec_shard_finish")
+
+
+def spec_check_bounded_wait(status):
+    """Launch a warp whose bounded mbarrier wait has nothing to wait for: after
+    about a second it gives up and sets ERR_TIMEOUT in `status` (int32 [1])."""
+    _check(library().spec_check_bounded_wait(_ptr(status), _stream(None)), "spec_check_bounded_wait")
 
 
 def spec_profile_stream_pass(before=None, after=None):

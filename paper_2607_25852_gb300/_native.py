@@ -28,6 +28,7 @@ SIGNATURES = {
                                 _P, _P, _P, _P, _P, _P, _P]),
     "spec_commit": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P]),
     "spec_profile_stream_pass": (_I, [_P, _P]),
+    "spec_check_bounded_wait": (_I, [_P, _P]),
     "spec_draft_workspace": (_SZ, [_I, _I, _I]),
     "spec_draft": (_I, [_P, _I, _I, _I, _I, ctypes.c_float, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "spec_markov_workspace": (_SZ, [_I, _I, _I, _I]),

@@ -784,6 +784,19 @@ __global__ void __launch_bounds__(128) markov_begin_kernel(const MarkovLaunch p)
     p.E[(size_t)e * p.r + j] = (i < p.B && !bad) ? p.W1[(size_t)x * p.r + j] : __float2bfloat16(0.0f);
 }
 
+// One warp waits on an mbarrier that nothing arrives at: the bounded wait
+// gives up and reports SPEC_ERR_TIMEOUT (spec_check_bounded_wait).
+__global__ void __launch_bounds__(32) bounded_wait_check_kernel(int32_t* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0u, status);
+  __syncwarp();
+}
+
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
@@ -919,4 +932,11 @@ extern "C" int spec_markov_draft(const void* U, int u_dtype, const void* W1, con
   }
   if (err != cudaSuccess || cudaGetLastError() != cudaSuccess) return SPEC_ERR_CUDA;
   return SPEC_OK;
+}
+
+extern "C" int spec_check_bounded_wait(int32_t* status, cudaStream_t stream) {
+  spec::NvtxRange range("spec_check_bounded_wait");
+  if (!status) return SPEC_ERR_INVALID_ARG;
+  spec::bounded_wait_check_kernel<<<1, 32, 0, stream>>>(status);
+  return cudaGetLastError() == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }

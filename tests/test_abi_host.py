@@ -95,6 +95,7 @@ def test_argument_errors_return_before_any_launch(lib):
     assert c(2, 2, dummy, dummy, H=0) == 1
     assert c(2, 2, dummy, dummy, dt=3) == 1
     assert lib.spec_profile_stream_pass(dummy, None) == 1
+    assert lib.spec_check_bounded_wait(None, stream) == 1  # no status word
 
 
 def test_shard_workspace_and_argument_errors(lib):
