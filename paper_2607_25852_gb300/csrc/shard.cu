@@ -619,11 +619,16 @@ __global__ void __launch_bounds__(kSampleThreads, 4) shard_sample_kernel(const S
 // ---------------------------------------------------------------------------
 // spec_shard_finish: one warp per request.
 // ---------------------------------------------------------------------------
-// Candidate block b with weight sum W (summed over its parts): key E_b / W.
-__device__ __forceinline__ void finish_block(KeyState& best, int& y, int b, float W, int y_part, const RaceArgs& a) {
-  if (!(W > 0.0f)) return;
+// The level-1 race word of block b.
+__device__ __forceinline__ uint32_t block_word(int b, const RaceArgs& a) {
   const uint4 r = philox(draw_counter(a.position, a.req, SPEC_PURPOSE_SAMPLE, (uint32_t)(b >> 2)), a.k0, a.k1);
-  const uint32_t word = (b & 3) == 0 ? r.x : (b & 3) == 1 ? r.y : (b & 3) == 2 ? r.z : r.w;
+  return (b & 3) == 0 ? r.x : (b & 3) == 1 ? r.y : (b & 3) == 2 ? r.z : r.w;
+}
+
+// Candidate block b with weight sum W (summed over its parts) and race word
+// `word`: key E_b / W.
+__device__ __forceinline__ void finish_block(KeyState& best, int& y, int b, float W, int y_part, uint32_t word) {
+  if (!(W > 0.0f)) return;
   const KeyState k{race_key(race_m(word), W), b};
   if (key_better(k, best)) {
     best = k;
@@ -637,6 +642,7 @@ constexpr int kFinishWarps = 4;
 
 __global__ void __launch_bounds__(32 * kFinishWarps) shard_finish_kernel(const ShardLaunch p) {
   __shared__ ShardRace sh_rec[kFinishWarps][32];
+  __shared__ uint32_t sh_word[kFinishWarps][32][2];  // the race words of the records' cut blocks
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * kFinishWarps + warp;
   pdl_wait_prerequisites();
@@ -657,6 +663,7 @@ __global__ void __launch_bounds__(32 * kFinishWarps) shard_finish_kernel(const S
   int yr = -1, yq = -1;
   // cut blocks: the parts of one block are adjacent in shard order
   int cur = INT_MAX;
+  uint32_t cur_word = 0;
   float Wr = 0.0f, Wp = 0.0f;
   KeyState er{INFINITY, INT_MAX}, ep{INFINITY, INT_MAX};
   for (int s0 = 0; s0 < p.S; s0 += 32) {
@@ -666,6 +673,13 @@ __global__ void __launch_bounds__(32 * kFinishWarps) shard_finish_kernel(const S
       uint4* dst = reinterpret_cast<uint4*>(&sh_rec[warp][lane]);
 #pragma unroll
       for (int w = 0; w < (int)(sizeof(ShardRace) / 16); ++w) dst[w] = src[w];
+      // the race words of this record's cut blocks, a lane per record (lane
+      // 0 then merges the records in shard order)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int b = sh_rec[warp][lane].part[h].blk;
+        sh_word[warp][lane][h] = b != INT_MAX ? block_word(b, a) : 0u;
+      }
     }
     __syncwarp();
     if (lane != 0) continue;
@@ -685,10 +699,11 @@ __global__ void __launch_bounds__(32 * kFinishWarps) shard_finish_kernel(const S
         if (pt.blk == INT_MAX) continue;
         if (pt.blk != cur) {
           if (cur != INT_MAX) {
-            finish_block(r, yr, cur, Wr, er.idx, a);
-            finish_block(q, yq, cur, Wp, ep.idx, a);
+            finish_block(r, yr, cur, Wr, er.idx, cur_word);
+            finish_block(q, yq, cur, Wp, ep.idx, cur_word);
           }
           cur = pt.blk;
+          cur_word = sh_word[warp][s - s0][h];
           Wr = Wp = 0.0f;
           er = ep = KeyState{INFINITY, INT_MAX};
         }
@@ -702,8 +717,8 @@ __global__ void __launch_bounds__(32 * kFinishWarps) shard_finish_kernel(const S
   }
   if (lane != 0) return;
   if (cur != INT_MAX) {
-    finish_block(r, yr, cur, Wr, er.idx, a);
-    finish_block(q, yq, cur, Wp, ep.idx, a);
+    finish_block(r, yr, cur, Wr, er.idx, cur_word);
+    finish_block(q, yq, cur, Wp, ep.idx, cur_word);
   }
   const int y = r.idx != INT_MAX ? yr : yq;
   int32_t* tok = p.out_tokens + (size_t)i * (p.K + 1);
