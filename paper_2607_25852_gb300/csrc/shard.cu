@@ -409,25 +409,37 @@ __device__ __forceinline__ KeyState shard_level2(const ShardLaunch& p, int mode,
   return race_level2<T, kWeightP>(row, qrow, p.q_dtype, vend, p.v_begin, b, ra, sh);
 }
 
-// Sum over the CTA (kSampleThreads threads; result in every thread).
-__device__ __forceinline__ float cta_sum(float x, float* sh) {
+// The lowest keys a and b over the CTA in one exchange (results in thread 0;
+// sh: 2 x kSampleThreads / 32 slots).
+__device__ __forceinline__ void cta_min_key2(KeyState& a, KeyState& b, KeyState* sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
-  if (lane == 0) sh[warp] = x;
+  for (int o = 16; o > 0; o >>= 1) {
+    const KeyState oa{__shfl_xor_sync(0xFFFFFFFFu, a.key, o), __shfl_xor_sync(0xFFFFFFFFu, a.idx, o)};
+    const KeyState ob{__shfl_xor_sync(0xFFFFFFFFu, b.key, o), __shfl_xor_sync(0xFFFFFFFFu, b.idx, o)};
+    if (key_better(oa, a)) a = oa;
+    if (key_better(ob, b)) b = ob;
+  }
+  if (lane == 0) {
+    sh[warp] = a;
+    sh[kSampleThreads / 32 + warp] = b;
+  }
   __syncthreads();
-  float t = 0.0f;
-#pragma unroll
-  for (int k = 0; k < kSampleThreads / 32; ++k) t += sh[k];
+  if (threadIdx.x == 0)
+    for (int k = 0; k < kSampleThreads / 32; ++k) {
+      if (key_better(sh[k], a)) a = sh[k];
+      if (key_better(sh[kSampleThreads / 32 + k], b)) b = sh[kSampleThreads / 32 + k];
+    }
   __syncthreads();
-  return t;
 }
 
 // The shard's part [lo, hi) of block b (one entry per thread): the part's
-// weight sums and lowest entry keys.  Result in thread 0.
+// weight sums (a warp butterfly, then the warps' sums in warp order) and
+// lowest entry keys, from one exchange over the CTA.  Result in thread 0.
 template <typename T>
 __device__ ShardPart shard_part(const ShardLaunch& p, int mode, const T* row, const void* qrow, int b, int lo, int hi,
                                 const RaceArgs& ra, KeyState* sh_key, float* sh_f) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int v = b * kRaceBlock + (int)threadIdx.x;
   float w = 0.0f, wp = 0.0f;
   KeyState er{INFINITY, INT_MAX}, ep{INFINITY, INT_MAX};
@@ -447,10 +459,25 @@ __device__ ShardPart shard_part(const ShardLaunch& p, int mode, const T* row, co
   }
   ShardPart out;
   out.blk = b;
-  out.w_r = cta_sum(w, sh_f);
-  out.w_p = cta_sum(wp, sh_f);
-  er = cta_min_key(er, sh_key);
-  ep = cta_min_key(ep, sh_key);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    w += __shfl_xor_sync(0xFFFFFFFFu, w, o);
+    wp += __shfl_xor_sync(0xFFFFFFFFu, wp, o);
+  }
+  if (lane == 0) {
+    sh_f[warp] = w;
+    sh_f[kSampleThreads / 32 + warp] = wp;
+  }
+  cta_min_key2(er, ep, sh_key);  // its barriers also publish sh_f
+  float t = 0.0f, tp = 0.0f;
+#pragma unroll
+  for (int k = 0; k < kSampleThreads / 32; ++k) {
+    t += sh_f[k];
+    tp += sh_f[kSampleThreads / 32 + k];
+  }
+  __syncthreads();  // sh_f is reused by the next part
+  out.w_r = t;
+  out.w_p = tp;
   out.ek_r = er.key;
   out.ey_r = er.idx;
   out.ek_p = ep.key;
@@ -489,8 +516,8 @@ template <typename T>
 __global__ void __launch_bounds__(kSampleThreads, 4) shard_sample_kernel(const ShardLaunch p) {
   __shared__ int sh_last, sh_b, sh_bp;
   __shared__ float sh_kb, sh_kbp;
-  __shared__ KeyState sh_red[kSampleThreads / 32];
-  __shared__ float sh_f[kSampleThreads / 32];
+  __shared__ KeyState sh_red[2 * (kSampleThreads / 32)];
+  __shared__ float sh_f[2 * (kSampleThreads / 32)];
   const int i = blockIdx.x / p.NCS;
   const int cs = blockIdx.x - i * p.NCS;
   pdl_wait_prerequisites();
@@ -529,8 +556,7 @@ __global__ void __launch_bounds__(kSampleThreads, 4) shard_sample_kernel(const S
     shard_level1<T, kWeightExcl, true>(p, row, qrow, q_first, q_end, ra, best, best_p);
   else
     shard_level1<T, kWeightP, false>(p, row, qrow, q_first, q_end, ra, best, best_p);
-  best = cta_min_key(best, sh_red);
-  if (mode != kWeightP) best_p = cta_min_key(best_p, sh_red);
+  cta_min_key2(best, best_p, sh_red);
   // ---- the cut blocks at the shard's ends: the first and the last chunk's
   // CTA compute the shard's part of each before arriving ----
   const int hb = p.v_begin / kRaceBlock;   // block holding the first column
