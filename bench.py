@@ -698,8 +698,9 @@ def run_sharded(args):
     """Vocabulary-sharded verification (the target's TP layout) with the S
     shards on this one GPU: the whole round (S x stats, decide, S x sample,
     finish; the records written side by side in place of the all-gathers),
-    and the per-rank critical path (shard 0's stats and sample, decide,
-    finish), each call timed alone."""
+    and the per-rank critical path (stats, decide, sample, finish), each call
+    timed in a loop of back-to-back calls over the S shards and once alone
+    after an L2 flush."""
     import torch
     import paper_2607_25852_gb300 as spec
     from paper_2607_25852_gb300.sharded import ShardedRound, even_bounds
