@@ -10,7 +10,7 @@ hidden rows H=7168 bf16):
     spec_commit    packing of the committed tokens and hidden rows
 
 value = verified positions per second (rows verified / step time), inputs
-resident in HBM.  The logits alone (437.6 MB) exceed L2 (126 MB), so no L2
+resident in HBM.  The logits alone (437.6 MB) exceed L2 (129 MB), so no L2
 flush is needed between steps.  The JSON line also carries the roofline of the
 vocabulary-streaming kernel, clocks sampled during the timed region, an
 end-to-end number through the same public API with host (pinned) buffers, and
